@@ -1,0 +1,216 @@
+/*
+ * hsa.h -- C ABI of libhsa, the GB300 (sm_103a) hot path of Heterogeneous Step
+ * Allocation (HSA), a training-free step-skipping scheme for video diffusion
+ * transformers (arXiv 2605.06892).
+ *
+ * One denoising iteration i of an HSA layer runs, in order:
+ *   hsa_partition_active   active set A_i from the token groups     (Sec. 2.2, 2.5)
+ *   hsa_gather_active      rows of A_i entering the block            (Sec. 2.3, step 1)
+ *   hsa_kv_sync_scatter    fresh K/V of A_i into the layer's cache   (Sec. 2.3, step 2)
+ *   hsa_active_attention   |A_i| queries against all N cached keys   (Sec. 2.3, step 3)
+ *   hsa_cached_euler       all N latents advanced by one Euler step  (Sec. 2.4, Eq. 6)
+ * and, once per sample, hsa_partition assigns tokens to step-budget groups
+ * from a per-token statistic (Sec. 2.2 Eq. 3, Eq. 5; App. B, Eq. 7).
+ *
+ * Conventions for every call below:
+ *  - Pointers named as device pointers must be device (or managed) memory of
+ *    the current CUDA device; the caller owns all memory.  Host pointers are
+ *    read before the call returns.  The library allocates nothing.
+ *  - Work is enqueued on `stream` (NULL = the legacy default stream) and the
+ *    call returns without waiting for it.  Argument checks happen on the host
+ *    before any launch; a failed check launches nothing.
+ *  - Errors that only the GPU can see (an index out of range, a non-finite
+ *    statistic, a pipeline wait that ran out) do not fault the GPU: the kernel
+ *    skips the offending access, records the error in a per-device word, and
+ *    hsa_get_device_error() reports it.
+ *  - Return values are hsa_status codes (0 = success, negative = error), or a
+ *    documented non-negative count.
+ *  - Token tensors are row-major with the token index outermost: a [N, H, D]
+ *    tensor stores element (n, h, d) at offset (n*H + h)*D + d.
+ */
+#ifndef HSA_H
+#define HSA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+struct CUstream_st;
+typedef struct CUstream_st *hsa_stream_t;
+
+typedef enum {
+    HSA_BF16 = 0,   /* bfloat16 storage, fp32 accumulation */
+    HSA_F32 = 1     /* fp32 storage and arithmetic */
+} hsa_dtype;
+
+typedef enum {
+    HSA_OK = 0,
+    HSA_ERR_INVALID_ARG = -1,   /* null pointer, bad size, misaligned pointer */
+    HSA_ERR_NOT_DIVISOR = -2,   /* a step budget does not divide T (Eq. 5) */
+    HSA_ERR_BAD_COUNTS = -3,    /* group sizes negative or not summing to N */
+    HSA_ERR_UNSUPPORTED = -4,   /* shape outside the supported set */
+    HSA_ERR_NONFINITE = -5,     /* NaN or infinite statistic (device-side) */
+    HSA_ERR_INDEX = -6,         /* index or group id out of range (device-side) */
+    HSA_ERR_TIMEOUT = -7,       /* a bounded pipeline wait ran out (device-side) */
+    HSA_ERR_CUDA = -8,          /* a CUDA runtime call or launch failed */
+    HSA_ERR_WORKSPACE = -9      /* workspace missing, too small or misaligned */
+} hsa_status;
+
+/* Static string for a status code. */
+const char *hsa_status_string(int status);
+
+/* Library ABI version, currently 1. */
+int hsa_version(void);
+
+/* ------------------------------------------------------------ host helpers */
+
+/* Checks step budgets and group sizes against Sec. 2.2: budgets[0] == T (the
+ * baseline group G_1), budgets non-increasing, each a positive divisor of T
+ * (Eq. 5); counts[k] >= 0 with sum N (counts may be NULL to skip that part).
+ * Host only.  Returns HSA_OK, HSA_ERR_INVALID_ARG, HSA_ERR_NOT_DIVISOR or
+ * HSA_ERR_BAD_COUNTS. */
+int hsa_check_budgets(int T, const int *budgets, const int *counts, int K, int N);
+
+/* Margin m = floor((1 - k) T / 2) of the phase-aware caching window (Sec. 2.5)
+ * for k = window_pct / 100, in integer arithmetic.  Iterations i < m and
+ * i > T - m - 1 run every token.  Returns m, or HSA_ERR_INVALID_ARG when
+ * window_pct is outside [0, 100] or T < 1.  Host only. */
+int hsa_window_margin(int T, int window_pct);
+
+/* |A_i| from the group sizes: the sum of counts[k] over the groups active at
+ * iteration iter (group k is active iff iter mod (T / budgets[k]) == 0, or
+ * iter lies outside the caching window).  Host only, no device access, so a
+ * caller can size buffers without synchronising.  Negative on bad input. */
+int hsa_active_count(const int *budgets, const int *counts, int K, int T,
+                     int iter, int window_pct);
+
+/* Noise levels sigma_0 = 1 > sigma_1 > ... > sigma_T = 0 of the Euler solver
+ * (Sec. 2.1, Eq. 2), computed in fp64 into the host array sigma[T + 1]:
+ * t_i = 1 - i/T and sigma_i = shift*t_i / (1 + (shift - 1) t_i); shift = 1
+ * gives the linear schedule.  The step of iteration i is sigma_{i+1} - sigma_i
+ * (negative).  Host only. */
+int hsa_sigma_schedule(int T, double shift, double *sigma);
+
+/* ------------------------------------------------------------- a1 partition */
+
+/* Bytes of device workspace hsa_partition needs for N tokens (0 for N == 0). */
+size_t hsa_partition_workspace_bytes(int N);
+
+/* Token partition (Sec. 2.2 Eq. 3) by the dynamic selection rule (App. B,
+ * Eq. 7): tokens are ranked by stat ascending, ties broken by the lower token
+ * index (-0 and +0 are equal); the counts[K-1] lowest go to group K-1 (the
+ * smallest budget), the next counts[K-2] to group K-2, ..., the counts[0]
+ * highest to group 0, the baseline group with budgets[0] == T.
+ *   stat       device, fp32 [N]: per-token statistic (e.g. the mean L1
+ *              relative change of the velocity, Eq. 7, or any score).
+ *   budgets,   host, int [K]: step budget s_k and size |G_k| of each group,
+ *   counts     checked as hsa_check_budgets does; 1 <= K <= 32.
+ *   group_of   device, int32 [N], written: group id in [0, K) per token.
+ *   workspace  device, >= hsa_partition_workspace_bytes(N) bytes, 256-byte
+ *              aligned; overwritten.  Must not overlap stat or group_of.
+ * A NaN or infinite statistic is reported as HSA_ERR_NONFINITE by
+ * hsa_get_device_error; group_of is then unspecified. */
+int hsa_partition(const float *stat, int N, int T, const int *budgets,
+                  const int *counts, int K, int32_t *group_of, void *workspace,
+                  size_t workspace_bytes, hsa_stream_t stream);
+
+/* ---------------------------------------------------- a2 active set per step */
+
+/* Active set A_i (Sec. 2.3; Fig. 1): token n is active at iteration iter iff
+ * iter mod (T / budgets[group_of[n]]) == 0 (Sec. 2.2) or iter is outside the
+ * caching window of window_pct percent (Sec. 2.5; 100 = no window).
+ *   group_of  device, int32 [N] in [0, K).
+ *   idx       device, int32 [>= |A_i|], written: active token ids ascending.
+ *   pos       device, int32 [N] or NULL, written: rank of n in idx, or -1.
+ * |A_i| is hsa_active_count(...) of the same groups, known on the host.  A
+ * group id outside [0, K) is reported as HSA_ERR_INDEX (that token is then
+ * treated as skipped). */
+int hsa_partition_active(const int32_t *group_of, int N, int T,
+                         const int *budgets, int K, int iter, int window_pct,
+                         int32_t *idx, int32_t *pos, hsa_stream_t stream);
+
+/* --------------------------------------------------------------- a3 gather */
+
+/* dst[j, :] = src[idx[j], :] for j < n_active: the rows of the active tokens
+ * that enter the transformer block (Sec. 2.3, step 1).
+ *   src       device, [N, row_bytes] (any element type).
+ *   row_bytes row size in bytes, a positive multiple of 16; src and dst
+ *             16-byte aligned.
+ *   idx       device, int32 [n_active], values in [0, N).
+ *   dst       device, [n_active, row_bytes], written.
+ * An index outside [0, N) leaves its dst row untouched (HSA_ERR_INDEX). */
+int hsa_gather_active(const void *src, size_t row_bytes, int N,
+                      const int32_t *idx, int n_active, void *dst,
+                      hsa_stream_t stream);
+
+/* ------------------------------------------------------ a4 KV-cache scatter */
+
+/* KV-cache synchronisation (Sec. 2.3, step 2): k_cache[idx[j]] = k_fresh[j]
+ * and v_cache[idx[j]] = v_fresh[j] for j < n_active, one launch for both;
+ * rows of skipped tokens are left untouched.
+ *   k_cache, v_cache  device, [N, H, D] of dtype, updated in place.
+ *   k_fresh, v_fresh  device, [n_active, H, D] of dtype (K/V of A_i).
+ *   idx               device, int32 [n_active], distinct values in [0, N)
+ *                     (A_i never repeats a token; repeated ids race).
+ * H*D*sizeof(dtype) must be a multiple of 16 bytes and every pointer 16-byte
+ * aligned.  An index outside [0, N) skips its row (HSA_ERR_INDEX). */
+int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_fresh,
+                        const void *v_fresh, const int32_t *idx, int n_active,
+                        int N, int H, int D, hsa_dtype dtype,
+                        hsa_stream_t stream);
+
+/* -------------------------------------------------- a5 active attention */
+
+/* Full-context attention of the active queries (Sec. 2.3, step 3; Sec. 2.1
+ * "Self-attention"), per head h and active row j:
+ *   out[j, h, :] = sum_n softmax_n(scale * <q_{r,h}, k_{n,h}>) v_{n,h}
+ * over all N cached keys, with r = q_idx[j] when q_idx is given (q is then
+ * [N, H, D] and rows are read by index) or r = j (q is compact
+ * [n_active, H, D]).  No mask; scale <= 0 selects 1/sqrt(D).  The cost is
+ * O(|A_i| N) instead of O(N^2).
+ *   k_cache, v_cache  device, [N, H, D] of dtype.
+ *   out               device, [n_active, H, D] of dtype, written.
+ * Supported: D in {64, 128}; H >= 1; 1 <= N < 2^31; 0 <= n_active.
+ * HSA_BF16 runs on the tensor cores (tcgen05, fp32 accumulation); HSA_F32
+ * runs in fp32 on the CUDA cores.  Pointers must be 16-byte aligned.  A q_idx
+ * entry outside [0, N) yields a zero query row (HSA_ERR_INDEX). */
+int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
+                         const void *k_cache, const void *v_cache, int N, int H,
+                         int D, float scale, void *out, hsa_dtype dtype,
+                         hsa_stream_t stream);
+
+/* ------------------------------------------------------- a6 cached Euler */
+
+/* Cached Euler update (Sec. 2.4, Eq. 6) of all N tokens in one pass: when
+ * pos[n] >= 0 the velocity cache takes the fresh velocity,
+ * v_cache[n] = v_fresh[pos[n]]; then x[n] = fma(v_cache[n], dsigma, x[n])
+ * (fp32, one rounding per element), dsigma = sigma_{i+1} - sigma_i.
+ *   x, v_cache  device, fp32 [N, C], updated in place.
+ *   v_fresh     device, fp32 [n_active, C] (velocities of A_i) or NULL.
+ *   pos         device, int32 [N] (as written by hsa_partition_active) or
+ *               NULL; both NULL = no refresh.
+ *   n_fresh     rows of v_fresh; a pos value outside [-1, n_fresh) is
+ *               treated as -1 and reported as HSA_ERR_INDEX.
+ * C must be a positive multiple of 4 and the pointers 16-byte aligned. */
+int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
+                     const int32_t *pos, int n_fresh, int N, int C, float dsigma,
+                     hsa_stream_t stream);
+
+/* ------------------------------------------------------------------ errors */
+
+/* Waits for `stream`, then reports and clears the device-side errors recorded
+ * on the current device since the last call: HSA_ERR_TIMEOUT if a bounded wait
+ * ran out, else HSA_ERR_NONFINITE, else HSA_ERR_INDEX, else HSA_OK; or
+ * HSA_ERR_CUDA if the wait itself failed.  The word is per device, shared by
+ * every stream and thread. */
+int hsa_get_device_error(hsa_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HSA_H */

@@ -1,0 +1,681 @@
+// Active-query full-context attention (Sec. 2.3, step 3): the |A_i| active
+// queries attend to all N rows of the layer's KV cache, O(|A_i| N) work.
+//
+// bf16 path: one CTA owns 256 active query rows (two 128-row Q tiles) of one
+// head and streams every 128-key tile of that head's cache through shared
+// memory.  Warp roles:
+//   warp 0      TMA producer: K and V tiles of the head, 128-byte swizzled,
+//               into a ring of shared-memory slots (rows >= N are zero-filled).
+//   warp 1      tensor-core issuer (one thread): S_t = Q_t K^T into TMEM and
+//               O_t += P_t V from TMEM P and shared V, tcgen05.mma kind::f16.
+//   warps 2-5   softmax of Q tile 0, warps 6-9 softmax of Q tile 1: each
+//               thread owns one query row (its TMEM lane; a warp may only
+//               reach the lane quarter warp%4), reads its S row,
+//               keeps the running maximum and sum, writes P as bf16 back into
+//               the S columns, and at the end normalises O and stores it.
+//   all warps   load the 256 query rows once, by index, into swizzled smem.
+// The two Q tiles ping-pong: while one softmax group works on its scores the
+// tensor core runs the other tile's MMAs.  The running maximum is only moved
+// (and O rescaled in TMEM) when it grows by more than 2^8, so most iterations
+// skip the rescale; the final division by the running sum makes the result
+// exact whatever maximum was used.
+// Every mbarrier wait is bounded in time; on a timeout the kernel records
+// HSA_ERR_TIMEOUT, stops issuing work, drains its own copies and MMAs, frees
+// TMEM and returns.
+//
+// fp32 path: CUDA-core flash loop with K/V tiles in shared memory.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+
+#include <atomic>
+#include <cmath>
+
+#include "hsa_internal.cuh"
+
+namespace hsa {
+namespace {
+
+// ----------------------------------------------------------- PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(b)), "r"(count)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(b)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(b)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_test(uint64_t *b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(b)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// About one second at the GB300 clock.
+constexpr long long kWaitCycles = 2000000000LL;
+
+// Bounded wait on phase `parity` of barrier b.  Gives up when the time runs
+// out (records the timeout and raises the CTA's abort flag) or, if
+// `honor_abort`, as soon as another role has raised the abort flag.
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
+                                          unsigned *err, bool honor_abort = true) {
+  if (mbar_test(b, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_test(b, parity)) return true;
+    if (honor_abort && *abort_flag) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      set_error(err, kErrTimeout);
+      *abort_flag = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar,
+                                            int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(map), "r"(smem_addr(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05), 128-byte swizzle.  For a
+// K-major operand only the stride between 8-row groups (sbo) matters; for an
+// MN-major operand lbo is the stride between 64-element column chunks.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return (uint64_t)((saddr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// Instruction descriptor of kind::f16 with bf16 A/B, fp32 accumulator.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)b_mn_major << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t id,
+                                       uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(id), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t id,
+                                       uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
+      "r"(a_tmem), "l"(b), "r"(id), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t *b) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_addr(b))
+      : "memory");
+}
+
+// 32 consecutive TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+      "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// ------------------------------------------------------ tcgen05 kernel
+
+constexpr int kBM = 128;         // query rows per Q tile (= TMEM lanes)
+constexpr int kQT = 2;           // Q tiles per CTA
+constexpr int kBN = 128;         // keys per K/V tile
+constexpr int kTcThreads = 320;  // 10 warps
+constexpr int kTmemCols = 512;
+constexpr float kRescaleLog2 = 8.0f;   // lazy rescale threshold, log2 units
+
+template <int D>
+struct TcCfg {
+  static constexpr int kTileBytes = kBM * D * 2;            // one Q, K or V tile
+  static constexpr int kChunks = D / 64;                    // 128-byte column chunks
+  static constexpr int kStages = D == 128 ? 4 : 8;          // K/V ring slots
+  static constexpr int kSmem = (kQT + kStages) * kTileBytes + 1024;
+  static constexpr int kOCol0 = 256;                        // O_t at kOCol0 + t*D
+};
+
+struct TcArgs {
+  const __nv_bfloat16 *q;
+  const int32_t *q_idx;
+  __nv_bfloat16 *out;
+  unsigned *err;
+  int n_active, N, H, q_rows, n_kv_tiles;
+  float scale_log2;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, 1)
+attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+               const TcArgs a) {
+  using C = TcCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                            ~(uintptr_t)1023);
+  uint8_t *sQ = sm;
+  uint8_t *sKV = sm + kQT * C::kTileBytes;
+  __shared__ __align__(8) uint64_t bar_full[C::kStages], bar_empty[C::kStages];
+  __shared__ __align__(8) uint64_t bar_s[kQT], bar_p[kQT], bar_o;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y;
+  const int row0 = blockIdx.x * (kBM * kQT);
+  const int nT = a.n_kv_tiles;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_empty[s], 1);
+    }
+    for (int t = 0; t < kQT; ++t) {
+      mbar_init(&bar_s[t], 1);
+      mbar_init(&bar_p[t], kBM);
+    }
+    mbar_init(&bar_o, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_addr(&tmem_base_sh)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+
+  // ---- query rows, by index, into the two swizzled Q tiles (all threads)
+  {
+    constexpr int kVecPerRow = D / 8;                        // 16-byte vectors per row
+    const size_t row_stride = (size_t)a.H * D;
+    for (int i = threadIdx.x; i < kBM * kQT * kVecPerRow; i += kTcThreads) {
+      const int row = i / kVecPerRow, c = i % kVecPerRow;
+      const int grow = row0 + row;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (grow < a.n_active) {
+        const int src = a.q_idx ? __ldg(a.q_idx + grow) : grow;
+        if (src >= 0 && src < a.q_rows)
+          v = __ldg(reinterpret_cast<const uint4 *>(a.q + (size_t)src * row_stride +
+                                                    (size_t)h * D) + c);
+        else if (c == 0)
+          set_error(a.err, kErrIndex);
+      }
+      const int t = row / kBM, rr = row % kBM;
+      uint8_t *dst = sQ + t * C::kTileBytes + (c >> 3) * (kBM * 128) + rr * 128 +
+                     (((c & 7) ^ (rr & 7)) << 4);
+      *reinterpret_cast<uint4 *>(dst) = v;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = tmem_base_sh;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int issued = 0;
+      for (int L = 0; L < 2 * nT; ++L) {
+        const int slot = L % C::kStages, use = L / C::kStages;
+        if (use > 0 && !mbar_wait(&bar_empty[slot], (use - 1) & 1, &abort_flag, a.err)) break;
+        mbar_expect_tx(&bar_full[slot], C::kTileBytes);
+        const CUtensorMap *map = (L & 1) ? &tm_v : &tm_k;
+        uint8_t *dst = sKV + slot * C::kTileBytes;
+#pragma unroll
+        for (int c = 0; c < C::kChunks; ++c)
+          tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, (L >> 1) * kBN);
+        issued = L + 1;
+      }
+      // Drain: every issued copy has landed before the CTA may exit.
+      for (int L = issued > C::kStages ? issued - C::kStages : 0; L < issued; ++L)
+        mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err, false);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdS = idesc_bf16(kBM, kBN, 0);
+      constexpr uint32_t kIdO = idesc_bf16(kBM, D, 1);
+      const uint32_t q_base = smem_addr(sQ);
+      const uint32_t kv_base = smem_addr(sKV);
+      auto slot_addr = [&](int L) { return kv_base + (L % C::kStages) * C::kTileBytes; };
+      auto wait_full = [&](int L) {
+        return mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err);
+      };
+      // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
+      auto issue_s = [&](int t, int L) {
+        const uint32_t qa = q_base + t * C::kTileBytes, ka = slot_addr(L);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k) {
+          const uint32_t off = (k >> 2) * (kBM * 128) + (k & 3) * 32;
+          mma_ss(tmem + 128 * t, sdesc(qa + off, 16, 1024), sdesc(ka + off, 16, 1024), kIdS,
+                 k > 0);
+        }
+      };
+      // O_t += P_t V: P in TMEM (bf16 pairs in the S_t columns), V MN-major.
+      auto issue_o = [&](int t, int L, bool acc) {
+        const uint32_t va = slot_addr(L);
+#pragma unroll
+        for (int k = 0; k < kBN / 16; ++k)
+          mma_ts(tmem + C::kOCol0 + D * t, tmem + 128 * t + 8 * k,
+                 sdesc(va + k * 2048, kBN * 128, 1024), kIdO, (acc || k > 0) ? 1u : 0u);
+      };
+      bool ok = wait_full(0);
+      if (ok) {
+        fence_after();
+        issue_s(0, 0);
+        mma_commit(&bar_s[0]);
+        issue_s(1, 0);
+        mma_commit(&bar_s[1]);
+        mma_commit(&bar_empty[0]);
+      }
+      for (int j = 0; ok && j < nT; ++j) {
+        const int Lv = 2 * j + 1, Lk = 2 * j + 2;
+        const bool more = j + 1 < nT;
+        if (!(ok = wait_full(Lv))) break;
+        if (!(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err))) break;
+        fence_after();
+        issue_o(0, Lv, j > 0);
+        if (more) {
+          if (!(ok = wait_full(Lk))) break;
+          fence_after();
+          issue_s(0, Lk);
+          mma_commit(&bar_s[0]);
+        }
+        if (!(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err))) break;
+        fence_after();
+        issue_o(1, Lv, j > 0);
+        mma_commit(&bar_empty[Lv % C::kStages]);
+        if (more) {
+          issue_s(1, Lk);
+          mma_commit(&bar_s[1]);
+          mma_commit(&bar_empty[Lk % C::kStages]);
+        }
+      }
+      // Completes once every MMA issued above has finished (also on abort),
+      // so TMEM is quiet before it is freed.
+      mma_commit(&bar_o);
+      mbar_wait(&bar_o, 0, &abort_flag, a.err, false);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------ softmax / epilogue
+    const int t = (warp - 2) >> 2;
+    const int wq = warp & 3;                       // TMEM lane quarter of this warp
+    const int r = wq * 32 + lane;                  // row within the Q tile
+    const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
+    const uint32_t tS = tmem + lane_off + 128 * t;
+    const uint32_t tO = tmem + lane_off + C::kOCol0 + D * t;
+    const float sl2 = a.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nT; ++j) {
+      if (!(ok = mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err))) break;
+      fence_after();
+      const int valid = a.N - j * kBN;             // keys of this tile that exist
+      // Pass 1: row maximum over the 128 scores, 64 columns per TMEM read.
+      float mx = -INFINITY;
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        uint32_t raw[2][32];
+        tmem_ld32(tS + 64 * h2, raw[0]);
+        tmem_ld32(tS + 64 * h2 + 32, raw[1]);
+        tmem_wait_ld();
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float v = __uint_as_float(raw[c][i]);
+            mx = (64 * h2 + 32 * c + i < valid) ? fmaxf(mx, v) : mx;
+          }
+      }
+      const float m_new = fmaxf(m_run, mx * sl2);
+      if (j == 0) {
+        m_run = m_new;
+      } else {
+        const bool need = m_new > m_run + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
+          if (need) {
+            l_run *= alpha;
+            m_run = m_new;
+          }
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(tO + 32 * c, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+            tmem_st32(tO + 32 * c, o);
+          }
+          tmem_wait_st();
+        }
+      }
+      // Pass 2: p = 2^(s*scale*log2e - m), packed to bf16 pairs into the first
+      // 64 columns of S.  The 64 scores of half h2 are read before the P
+      // columns [32*h2, 32*h2+32) they overlap are written.
+      float rs = 0.f;
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        uint32_t raw[2][32];
+        tmem_ld32(tS + 64 * h2, raw[0]);
+        tmem_ld32(tS + 64 * h2 + 32, raw[1]);
+        tmem_wait_ld();
+        uint32_t pk[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int col = 64 * h2 + 2 * i;
+          const float s0 = __uint_as_float(raw[(2 * i) / 32][(2 * i) % 32]);
+          const float s1 = __uint_as_float(raw[(2 * i + 1) / 32][(2 * i + 1) % 32]);
+          const float p0 = col < valid ? fast_exp2(fmaf(s0, sl2, -m_run)) : 0.f;
+          const float p1 = col + 1 < valid ? fast_exp2(fmaf(s1, sl2, -m_run)) : 0.f;
+          rs += p0 + p1;
+          pk[i] = pack_bf16(p0, p1);
+        }
+        tmem_st32(tS + 32 * h2, pk);
+      }
+      l_run += rs;
+      tmem_wait_st();
+      fence_before();
+      mbar_arrive(&bar_p[t]);
+    }
+    if (ok && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
+      fence_after();
+      const int grow = row0 + t * kBM + r;
+      const float inv = 1.f / l_run;
+      __nv_bfloat16 *dst = a.out + ((size_t)grow * a.H + h) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tO + 32 * c, o);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          pk[i] = pack_bf16(__uint_as_float(o[2 * i]) * inv, __uint_as_float(o[2 * i + 1]) * inv);
+        if (grow < a.n_active) {
+          uint4 *d4 = reinterpret_cast<uint4 *>(dst + 32 * c);
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        }
+      }
+    }
+  }
+
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------ fp32 CUDA-core kernel
+
+constexpr int kF32Threads = 128;
+constexpr int kF32Keys = 32;
+
+// TPQ = D/32 threads cooperate on one query; thread slice s owns dimensions
+// s, s+TPQ, s+2*TPQ, ... so that the slices of one query hit distinct banks.
+template <int D>
+__global__ void __launch_bounds__(kF32Threads)
+attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
+                const float *__restrict__ kc, const float *__restrict__ vc, float *__restrict__ out,
+                int n_active, int N, int H, int q_rows, float scale, unsigned *err) {
+  constexpr int TPQ = D / 32;
+  constexpr int QPB = kF32Threads / TPQ;
+  __shared__ float sK[kF32Keys][D];
+  __shared__ float sV[kF32Keys][D];
+  const int h = blockIdx.y;
+  const int ql = threadIdx.x / TPQ, sl = threadIdx.x % TPQ;
+  const int j = blockIdx.x * QPB + ql;
+  const bool active = j < n_active;
+  float qv[32], o[32];
+  bool row_ok = false;
+  if (active) {
+    const int src = q_idx ? q_idx[j] : j;
+    row_ok = src >= 0 && src < q_rows;
+    if (!row_ok && sl == 0) set_error(err, kErrIndex);
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      qv[i] = row_ok ? q[((size_t)src * H + h) * D + sl + TPQ * i] : 0.f;
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) qv[i] = 0.f;
+  }
+#pragma unroll
+  for (int i = 0; i < 32; ++i) o[i] = 0.f;
+  float m = -INFINITY, l = 0.f;
+  for (int n0 = 0; n0 < N; n0 += kF32Keys) {
+    __syncthreads();
+    for (int e = threadIdx.x; e < kF32Keys * D / 4; e += kF32Threads) {
+      const int kk = e / (D / 4), d4 = e % (D / 4);
+      float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
+      if (n0 + kk < N) {
+        const size_t off = ((size_t)(n0 + kk) * H + h) * D;
+        kv = reinterpret_cast<const float4 *>(kc + off)[d4];
+        vv = reinterpret_cast<const float4 *>(vc + off)[d4];
+      }
+      reinterpret_cast<float4 *>(&sK[kk][0])[d4] = kv;
+      reinterpret_cast<float4 *>(&sV[kk][0])[d4] = vv;
+    }
+    __syncthreads();
+    float sc[kF32Keys];
+    float tmax = -INFINITY;
+#pragma unroll
+    for (int kk = 0; kk < kF32Keys; ++kk) {
+      float dot = 0.f;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) dot = fmaf(qv[i], sK[kk][sl + TPQ * i], dot);
+#pragma unroll
+      for (int o2 = 1; o2 < TPQ; o2 <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o2);
+      sc[kk] = (n0 + kk < N) ? dot * scale : -INFINITY;
+      tmax = fmaxf(tmax, sc[kk]);
+    }
+    const float m_new = fmaxf(m, tmax);
+    const float corr = expf(m - m_new);
+    l *= corr;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) o[i] *= corr;
+#pragma unroll
+    for (int kk = 0; kk < kF32Keys; ++kk) {
+      const float p = expf(sc[kk] - m_new);
+      l += p;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) o[i] = fmaf(p, sV[kk][sl + TPQ * i], o[i]);
+    }
+    m = m_new;
+  }
+  if (active) {
+    const float inv = 1.f / l;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) out[((size_t)j * H + h) * D + sl + TPQ * i] = o[i] * inv;
+  }
+}
+
+// -------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::atomic<PFN_cuTensorMapEncodeTiled_v12000> fn{nullptr};
+  PFN_cuTensorMapEncodeTiled_v12000 f = fn.load();
+  if (!f) {
+    cudaDriverEntryPointQueryResult q;
+    void *p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return nullptr;
+    f = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    fn.store(f);
+  }
+  return f;
+}
+
+// 2-D map over a [N, H*D] bf16 cache: boxes of 64 columns x 128 rows,
+// 128-byte swizzle, rows past N read as zero.
+bool make_kv_map(CUtensorMap *map, const void *base, int N, int H, int D) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)H * D, (cuuint64_t)N};
+  const cuuint64_t strides[1] = {(cuuint64_t)H * D * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kBN};
+  const cuuint32_t estride[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+             box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
+              const void *v_cache, int N, int H, float scale, void *out, cudaStream_t stream,
+              unsigned *err) {
+  using C = TcCfg<D>;
+  static std::atomic<int> configured[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return HSA_ERR_CUDA;
+  if (!configured[dev].load()) {
+    if (cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmem) != cudaSuccess)
+      return HSA_ERR_CUDA;
+    configured[dev].store(1);
+  }
+  CUtensorMap mk, mv;
+  if (!make_kv_map(&mk, k_cache, N, H, D) || !make_kv_map(&mv, v_cache, N, H, D))
+    return HSA_ERR_CUDA;
+  TcArgs a;
+  a.q = static_cast<const __nv_bfloat16 *>(q);
+  a.q_idx = q_idx;
+  a.out = static_cast<__nv_bfloat16 *>(out);
+  a.err = err;
+  a.n_active = n_active;
+  a.N = N;
+  a.H = H;
+  a.q_rows = q_idx ? N : n_active;
+  a.n_kv_tiles = (N + kBN - 1) / kBN;
+  a.scale_log2 = scale * 1.4426950408889634f;
+  const dim3 grid((n_active + kBM * kQT - 1) / (kBM * kQT), H);
+  attn_tc_kernel<D><<<grid, kTcThreads, C::kSmem, stream>>>(mk, mv, a);
+  return launch_status();
+}
+
+template <int D>
+int launch_f32(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
+               const void *v_cache, int N, int H, float scale, void *out, cudaStream_t stream,
+               unsigned *err) {
+  constexpr int QPB = kF32Threads / (D / 32);
+  const dim3 grid((n_active + QPB - 1) / QPB, H);
+  attn_f32_kernel<D><<<grid, kF32Threads, 0, stream>>>(
+      static_cast<const float *>(q), q_idx, static_cast<const float *>(k_cache),
+      static_cast<const float *>(v_cache), static_cast<float *>(out), n_active, N, H,
+      q_idx ? N : n_active, scale, err);
+  return launch_status();
+}
+
+}  // namespace
+}  // namespace hsa
+
+using namespace hsa;
+
+extern "C" int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
+                                    const void *k_cache, const void *v_cache, int N, int H,
+                                    int D, float scale, void *out, hsa_dtype dtype,
+                                    hsa_stream_t stream) {
+  if (n_active < 0 || N < 1 || H < 1) return HSA_ERR_INVALID_ARG;
+  if (dtype != HSA_BF16 && dtype != HSA_F32) return HSA_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return HSA_ERR_UNSUPPORTED;
+  if ((long long)H * D > (1LL << 24)) return HSA_ERR_UNSUPPORTED;
+  if (!q_idx && n_active > N) return HSA_ERR_INVALID_ARG;
+  if (n_active == 0) return HSA_OK;
+  if (!q || !k_cache || !v_cache || !out) return HSA_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
+    return HSA_ERR_INVALID_ARG;
+  if (!(scale > 0.f) || !std::isfinite(scale)) scale = 1.f / std::sqrt((float)D);
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  cudaStream_t s = (cudaStream_t)stream;
+  if ((long long)(n_active + kBM * kQT - 1) / (kBM * kQT) > 0x7fffffffLL) return HSA_ERR_UNSUPPORTED;
+  if (H > 65535) return HSA_ERR_UNSUPPORTED;
+  if (dtype == HSA_BF16)
+    return D == 128 ? launch_tc<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err)
+                    : launch_tc<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
+  return D == 128 ? launch_f32<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err)
+                  : launch_f32<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
+}

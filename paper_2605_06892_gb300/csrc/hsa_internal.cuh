@@ -1,0 +1,46 @@
+// Internal helpers shared by the libhsa translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "hsa.h"
+
+namespace hsa {
+
+// Device-side error word bits.  Kernels never trap: they skip the offending
+// access, set a bit here with atomicOr, and hsa_get_device_error() maps the
+// lowest set bit back to a status code.
+enum : unsigned {
+  kErrIndex = 1u << 0,
+  kErrNonfinite = 1u << 1,
+  kErrTimeout = 1u << 2,
+};
+
+// Device address of this device's error word (resolved once per device).
+unsigned *device_error_word();
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+
+inline int launch_status() {
+  return cudaGetLastError() == cudaSuccess ? HSA_OK : HSA_ERR_CUDA;
+}
+
+inline bool aligned16(const void *p) {
+  return (reinterpret_cast<uintptr_t>(p) & 15u) == 0;
+}
+
+__device__ __forceinline__ void set_error(unsigned *err, unsigned bit) {
+  atomicOr(err, bit);
+}
+
+// Number of lanes that cooperate on one row of `vecs` 16-byte vectors:
+// a power of two, at most 32.
+inline int lanes_per_row(long long vecs) {
+  int l = 1;
+  while (l < 32 && l < vecs) l <<= 1;
+  return l;
+}
+
+}  // namespace hsa

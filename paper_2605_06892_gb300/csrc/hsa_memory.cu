@@ -1,0 +1,221 @@
+// Memory-bound steps of the HSA iteration: gather of the active rows
+// (Sec. 2.3, step 1), KV-cache synchronisation scatter (Sec. 2.3, step 2) and
+// the cached Euler update (Sec. 2.4, Eq. 6).
+//
+// All three move whole token rows.  A row is split into 16-byte vectors and a
+// group of L lanes (L a power of two <= 32) of one warp cooperates on a row, so
+// a warp covers 32/L rows at once and every access is a coalesced 128-bit load
+// or store.  Each lane keeps up to kUnroll vectors in flight before storing.
+// The row index is read once per row by its lane group; indices are checked
+// against the row count and a bad one skips its row and sets the error word.
+#include "hsa_internal.cuh"
+
+namespace hsa {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 4;
+
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+
+// Row loop shared by gather and scatter: rows are handed out to lane groups
+// in a grid-stride loop; `map(j, s, d)` sets the source and destination row
+// pointers of row j, or returns false to skip the row.
+template <class RowMap>
+__device__ __forceinline__ void copy_rows(long long n_rows, int vecs, int lpr_log2,
+                                          RowMap map) {
+  const int L = 1 << lpr_log2;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> lpr_log2;                  // row slot within the warp
+  const int sl = lane & (L - 1);                     // lane within the row group
+  const int rows_per_warp = 32 >> lpr_log2;
+  const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+  for (long long j = warp * rows_per_warp + sub; j < n_rows; j += nwarps * rows_per_warp) {
+    const uint4 *s;
+    uint4 *d;
+    if (!map(j, s, d)) continue;
+    for (int v0 = sl; v0 < vecs; v0 += kUnroll * L) {
+      uint4 buf[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int v = v0 + u * L;
+        if (v < vecs) buf[u] = ld_stream(s + v);
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int v = v0 + u * L;
+        if (v < vecs) d[v] = buf[u];
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+gather_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
+              const int32_t *__restrict__ idx, int n_active, int N, int vecs,
+              int lpr_log2, unsigned *err) {
+  copy_rows(n_active, vecs, lpr_log2, [&](long long j, const uint4 *&s, uint4 *&d) {
+    const int r = __ldg(idx + j);
+    if (r < 0 || r >= N) {
+      set_error(err, kErrIndex);
+      return false;
+    }
+    s = src + (long long)r * vecs;
+    d = dst + j * vecs;
+    return true;
+  });
+}
+
+// Rows 0..n_active-1 are K rows, n_active..2*n_active-1 the V rows, so a warp
+// moves K and V rows of different tokens with the same code.
+__global__ void __launch_bounds__(kThreads)
+scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
+               const uint4 *__restrict__ kf, const uint4 *__restrict__ vf,
+               const int32_t *__restrict__ idx, int n_active, int N, int vecs,
+               int lpr_log2, unsigned *err) {
+  copy_rows(2LL * n_active, vecs, lpr_log2, [&](long long jj, const uint4 *&s, uint4 *&d) {
+    const bool is_v = jj >= n_active;
+    const long long j = is_v ? jj - n_active : jj;
+    const int r = __ldg(idx + j);
+    if (r < 0 || r >= N) {
+      if (!is_v) set_error(err, kErrIndex);
+      return false;
+    }
+    s = (is_v ? vf : kf) + j * vecs;
+    d = (is_v ? vc : kc) + (long long)r * vecs;
+    return true;
+  });
+}
+
+// x[n] = fma(vhat[n], dsigma, x[n]) with vhat[n] refreshed from
+// v_fresh[pos[n]] when pos[n] >= 0.  A row is C/4 float4 vectors.
+__global__ void __launch_bounds__(kThreads)
+euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
+             const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
+             int N, int vecs, int lpr_log2, float dsigma, int n_fresh_rows, unsigned *err) {
+  const int L = 1 << lpr_log2;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> lpr_log2;
+  const int sl = lane & (L - 1);
+  const int rows_per_warp = 32 >> lpr_log2;
+  const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+  for (long long n = warp * rows_per_warp + sub; n < N; n += nwarps * rows_per_warp) {
+    int p = pos ? __ldg(pos + n) : -1;
+    if (p >= n_fresh_rows) {
+      set_error(err, kErrIndex);
+      p = -1;
+    }
+    float4 *xr = x + n * vecs;
+    float4 *vr = vhat + n * vecs;
+    const float4 *src = p >= 0 ? v_fresh + (long long)p * vecs : vr;
+    for (int v0 = sl; v0 < vecs; v0 += kUnroll * L) {
+      float4 vb[kUnroll], xb[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int v = v0 + u * L;
+        if (v < vecs) {
+          vb[u] = src[v];
+          xb[u] = xr[v];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int v = v0 + u * L;
+        if (v < vecs) {
+          if (p >= 0) vr[v] = vb[u];
+          float4 o;
+          o.x = __fmaf_rn(vb[u].x, dsigma, xb[u].x);
+          o.y = __fmaf_rn(vb[u].y, dsigma, xb[u].y);
+          o.z = __fmaf_rn(vb[u].z, dsigma, xb[u].z);
+          o.w = __fmaf_rn(vb[u].w, dsigma, xb[u].w);
+          xr[v] = o;
+        }
+      }
+    }
+  }
+}
+
+// Grid for n_rows rows handled by lane groups of size L: enough warps to give
+// every SM a full complement of resident threads, no more than the rows need.
+int grid_for(long long n_rows, int L) {
+  const long long rows_per_block = (long long)(kThreads / 32) * (32 / L);
+  long long blocks = (n_rows + rows_per_block - 1) / rows_per_block;
+  const long long cap = (long long)sm_count() * (2048 / kThreads);
+  if (blocks > cap) blocks = cap;
+  return (int)(blocks < 1 ? 1 : blocks);
+}
+
+int log2i(int L) {
+  int s = 0;
+  while ((1 << s) < L) ++s;
+  return s;
+}
+
+}  // namespace
+}  // namespace hsa
+
+using namespace hsa;
+
+extern "C" int hsa_gather_active(const void *src, size_t row_bytes, int N,
+                                 const int32_t *idx, int n_active, void *dst,
+                                 hsa_stream_t stream) {
+  if (N < 0 || n_active < 0 || row_bytes == 0 || (row_bytes & 15)) return HSA_ERR_INVALID_ARG;
+  if (n_active == 0) return HSA_OK;
+  if (!src || !dst || !idx || !aligned16(src) || !aligned16(dst)) return HSA_ERR_INVALID_ARG;
+  const long long vecs = (long long)(row_bytes / 16);
+  if (vecs > (1LL << 30)) return HSA_ERR_UNSUPPORTED;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const int L = lanes_per_row(vecs);
+  gather_kernel<<<grid_for(n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
+      (const uint4 *)src, (uint4 *)dst, idx, n_active, N, (int)vecs, log2i(L), err);
+  return launch_status();
+}
+
+extern "C" int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_fresh,
+                                   const void *v_fresh, const int32_t *idx, int n_active,
+                                   int N, int H, int D, hsa_dtype dtype,
+                                   hsa_stream_t stream) {
+  if (N < 0 || n_active < 0 || H < 1 || D < 1) return HSA_ERR_INVALID_ARG;
+  if (dtype != HSA_BF16 && dtype != HSA_F32) return HSA_ERR_INVALID_ARG;
+  const long long row_bytes = (long long)H * D * (dtype == HSA_BF16 ? 2 : 4);
+  if (row_bytes & 15) return HSA_ERR_UNSUPPORTED;
+  if (n_active == 0) return HSA_OK;
+  if (!k_cache || !v_cache || !k_fresh || !v_fresh || !idx) return HSA_ERR_INVALID_ARG;
+  if (!aligned16(k_cache) || !aligned16(v_cache) || !aligned16(k_fresh) || !aligned16(v_fresh))
+    return HSA_ERR_INVALID_ARG;
+  const long long vecs = row_bytes / 16;
+  if (vecs > (1LL << 30)) return HSA_ERR_UNSUPPORTED;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const int L = lanes_per_row(vecs);
+  scatter_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
+      (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
+      n_active, N, (int)vecs, log2i(L), err);
+  return launch_status();
+}
+
+extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
+                                const int32_t *pos, int n_fresh, int N, int C, float dsigma,
+                                hsa_stream_t stream) {
+  if (N < 0 || C < 4 || (C & 3) || n_fresh < 0) return HSA_ERR_INVALID_ARG;
+  if ((pos == nullptr) != (v_fresh == nullptr)) return HSA_ERR_INVALID_ARG;
+  if (N == 0) return HSA_OK;
+  if (!x || !v_cache || !aligned16(x) || !aligned16(v_cache)) return HSA_ERR_INVALID_ARG;
+  if (v_fresh && !aligned16(v_fresh)) return HSA_ERR_INVALID_ARG;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const int vecs = C / 4;
+  const int L = lanes_per_row(vecs);
+  euler_kernel<<<grid_for(N, L), kThreads, 0, (cudaStream_t)stream>>>(
+      (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, N, vecs, log2i(L), dsigma,
+      pos ? n_fresh : 0, err);
+  return launch_status();
+}

@@ -1,0 +1,338 @@
+// Token partition (Sec. 2.2, Eq. 3; App. B "dynamic token selection", Eq. 7)
+// and the per-iteration active set (Sec. 2.2 modular rule, Sec. 2.3, Sec. 2.5
+// caching window).
+//
+// Partition = a stable rank of the statistic.  Each fp32 value is mapped to an
+// unsigned key whose integer order is the float order (-0 folded onto +0), and
+// the (key, token) pairs are sorted by a least-significant-digit radix sort:
+// four passes of 8 bits, each pass a per-tile histogram, one exclusive scan of
+// the (digit, tile) counts in digit-major order, and a stable scatter.  Since
+// every pass is stable and the pairs start in token order, equal statistics
+// stay in token order, which is the tie rule.  Rank r then maps to its group.
+//
+// The active set needs no workspace: block b owns one chunk of tokens, counts
+// the active tokens of all earlier chunks itself (an L2-resident re-read that
+// is cheap at the token counts of a video DiT), then compacts its own chunk
+// with warp ballots and a block scan.
+#include <algorithm>
+
+#include "hsa_internal.cuh"
+
+namespace hsa {
+namespace {
+
+constexpr int kSortThreads = 256;
+constexpr int kItems = 16;                              // per thread per tile
+constexpr int kTile = kSortThreads * kItems;            // 4096 tokens
+constexpr int kWarps = kSortThreads / 32;
+constexpr int kWarpItems = kTile / kWarps;              // 512 consecutive tokens
+constexpr int kMaxGroups = 32;
+
+struct GroupStarts {
+  int start[kMaxGroups];   // first rank of group k (ranks ascend with the statistic)
+  int count[kMaxGroups];
+};
+
+size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+
+struct SortLayout {
+  size_t keys0, keys1, vals0, vals1, hist, total;
+  int tiles;
+};
+
+SortLayout sort_layout(int N) {
+  SortLayout L;
+  L.tiles = (N + kTile - 1) / kTile;
+  const size_t a = align256((size_t)N * 4);
+  L.keys0 = 0;
+  L.keys1 = a;
+  L.vals0 = 2 * a;
+  L.vals1 = 3 * a;
+  L.hist = 4 * a;
+  L.total = L.hist + align256((size_t)256 * L.tiles * 4);
+  return L;
+}
+
+__global__ void __launch_bounds__(kSortThreads)
+key_kernel(const float *__restrict__ stat, int N, uint32_t *__restrict__ keys,
+           int32_t *__restrict__ vals, unsigned *err) {
+  for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < N; n += gridDim.x * blockDim.x) {
+    const float f = stat[n];
+    uint32_t u = __float_as_uint(f);
+    if (!isfinite(f)) set_error(err, kErrNonfinite);
+    if (u == 0x80000000u) u = 0u;                          // -0 ranks with +0
+    keys[n] = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // float order as uint order
+    vals[n] = n;
+  }
+}
+
+__global__ void __launch_bounds__(kSortThreads)
+hist_kernel(const uint32_t *__restrict__ keys, int N, int shift, uint32_t *__restrict__ hist,
+            int tiles) {
+  __shared__ uint32_t h[256];
+  h[threadIdx.x] = 0;
+  __syncthreads();
+  const int base = blockIdx.x * kTile;
+#pragma unroll
+  for (int i = 0; i < kItems; ++i) {
+    const int n = base + i * kSortThreads + threadIdx.x;
+    if (n < N) atomicAdd(&h[(keys[n] >> shift) & 255u], 1u);
+  }
+  __syncthreads();
+  hist[threadIdx.x * tiles + blockIdx.x] = h[threadIdx.x];
+}
+
+// Exclusive scan, in place, of the 256*tiles counts in digit-major order, by
+// one block of 1024 threads, each owning a contiguous run.
+__global__ void __launch_bounds__(1024) scan_kernel(uint32_t *__restrict__ hist, int total) {
+  __shared__ uint32_t warp_sum[32];
+  const int per = (total + 1023) / 1024;
+  const int b = threadIdx.x * per;
+  const int e = min(total, b + per);
+  uint32_t s = 0;
+  for (int i = b; i < e; ++i) s += hist[i];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint32_t incl = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) warp_sum[w] = incl;
+  __syncthreads();
+  if (w == 0) {
+    uint32_t v = warp_sum[lane], inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += t;
+    }
+    warp_sum[lane] = inc - v;
+  }
+  __syncthreads();
+  uint32_t run = warp_sum[w] + incl - s;
+  for (int i = b; i < e; ++i) {
+    const uint32_t c = hist[i];
+    hist[i] = run;
+    run += c;
+  }
+}
+
+// Stable scatter of one tile.  Warp w owns tokens [w*512, w*512+512) of the
+// tile and walks them 32 at a time in order; lanes holding the same digit find
+// each other with __match_any_sync, so a token's rank among equal digits in
+// the tile is (earlier warps' count) + (this warp's running count) + (earlier
+// lanes of this step).
+__global__ void __launch_bounds__(kSortThreads)
+scatter_kernel(const uint32_t *__restrict__ kin, const int32_t *__restrict__ vin,
+               uint32_t *__restrict__ kout, int32_t *__restrict__ vout, int N, int shift,
+               const uint32_t *__restrict__ offsets, int tiles) {
+  __shared__ uint32_t cnt[kWarps][256];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  for (int d = threadIdx.x; d < kWarps * 256; d += kSortThreads) (&cnt[0][0])[d] = 0;
+  __syncthreads();
+  const unsigned lt_mask = (1u << lane) - 1u;
+  const int base = blockIdx.x * kTile + w * kWarpItems;
+  uint32_t key[kItems];
+  int32_t val[kItems];
+  uint32_t local[kItems];
+#pragma unroll
+  for (int it = 0; it < kItems; ++it) {
+    const int n = base + it * 32 + lane;
+    const bool valid = n < N;
+    key[it] = valid ? kin[n] : 0u;
+    val[it] = valid ? vin[n] : 0;
+    const uint32_t d = (key[it] >> shift) & 255u;
+    const unsigned peers = __match_any_sync(0xffffffffu, valid ? d : 256u + lane);
+    const uint32_t before = valid ? cnt[w][d] : 0u;
+    local[it] = before + __popc(peers & lt_mask);
+    __syncwarp();
+    if (valid && lane == __ffs(peers) - 1) cnt[w][d] = before + __popc(peers);
+    __syncwarp();
+  }
+  __syncthreads();
+  // exclusive prefix over warps, one digit per thread (blockDim == 256)
+  {
+    const int d = threadIdx.x;
+    uint32_t run = offsets[d * tiles + blockIdx.x];
+    for (int ww = 0; ww < kWarps; ++ww) {
+      const uint32_t c = cnt[ww][d];
+      cnt[ww][d] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int it = 0; it < kItems; ++it) {
+    const int n = base + it * 32 + lane;
+    if (n < N) {
+      const uint32_t d = (key[it] >> shift) & 255u;
+      const uint32_t p = cnt[w][d] + local[it];
+      kout[p] = key[it];
+      vout[p] = val[it];
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kSortThreads)
+assign_kernel(const int32_t *__restrict__ sorted_tokens, int N, int K, GroupStarts gs,
+              int32_t *__restrict__ group_of) {
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < N; r += gridDim.x * blockDim.x) {
+    int g = 0;
+    for (int k = 0; k < K; ++k)
+      if (r >= gs.start[k] && r < gs.start[k] + gs.count[k]) g = k;
+    group_of[sorted_tokens[r]] = g;
+  }
+}
+
+// ------------------------------------------------------------- active set
+
+constexpr int kActThreads = 1024;
+
+template <bool kVec>
+__global__ void __launch_bounds__(kActThreads)
+active_kernel(const int32_t *__restrict__ group_of, int N, int K, uint32_t mask, int chunk,
+              int32_t *__restrict__ idx, int32_t *__restrict__ pos, unsigned *err) {
+  __shared__ int warp_cnt[32];
+  __shared__ int block_base;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int start = blockIdx.x * chunk;
+  const int end = min(N, start + chunk);
+  auto act = [&](int g) -> int {
+    return (g >= 0 && g < K) ? (int)((mask >> g) & 1u) : 0;
+  };
+  // 1. active tokens before this chunk
+  int c = 0;
+  if (kVec) {
+    const int4 *g4 = reinterpret_cast<const int4 *>(group_of);
+    for (int i = threadIdx.x; i < start / 4; i += kActThreads) {
+      const int4 v = __ldg(g4 + i);
+      c += act(v.x) + act(v.y) + act(v.z) + act(v.w);
+    }
+  } else {
+    for (int i = threadIdx.x; i < start; i += kActThreads) c += act(__ldg(group_of + i));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) warp_cnt[w] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int s = 0;
+    for (int i = 0; i < kActThreads / 32; ++i) s += warp_cnt[i];
+    block_base = s;
+  }
+  __syncthreads();
+  int base = block_base;
+  // 2. compact this chunk, 1024 tokens at a time
+  for (int b0 = start; b0 < end; b0 += kActThreads) {
+    const int n = b0 + threadIdx.x;
+    int flag = 0;
+    if (n < end) {
+      const int g = group_of[n];
+      if (g < 0 || g >= K) set_error(err, kErrIndex);
+      flag = act(g);
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, flag);
+    __syncthreads();                                   // warp_cnt reuse
+    if (lane == 0) warp_cnt[w] = __popc(bal);
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int i = 0; i < kActThreads / 32; ++i) {
+      const int v = warp_cnt[i];
+      before += (i < w) ? v : 0;
+      total += v;
+    }
+    const int r = base + before + __popc(bal & ((1u << lane) - 1u));
+    if (n < end) {
+      if (flag) idx[r] = n;
+      if (pos) pos[n] = flag ? r : -1;
+    }
+    base += total;
+  }
+}
+
+}  // namespace
+}  // namespace hsa
+
+using namespace hsa;
+
+extern "C" size_t hsa_partition_workspace_bytes(int N) {
+  if (N <= 0) return 0;
+  return sort_layout(N).total;
+}
+
+extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets,
+                             const int *counts, int K, int32_t *group_of, void *workspace,
+                             size_t workspace_bytes, hsa_stream_t stream) {
+  if (!budgets || !counts || K < 1) return HSA_ERR_INVALID_ARG;
+  if (K > kMaxGroups) return HSA_ERR_UNSUPPORTED;
+  const int st = hsa_check_budgets(T, budgets, counts, K, N);
+  if (st != HSA_OK) return st;
+  if (N == 0) return HSA_OK;
+  if (!stat || !group_of) return HSA_ERR_INVALID_ARG;
+  const SortLayout L = sort_layout(N);
+  if (!workspace || workspace_bytes < L.total || (reinterpret_cast<uintptr_t>(workspace) & 255))
+    return HSA_ERR_WORKSPACE;
+  char *ws = static_cast<char *>(workspace);
+  uint32_t *keys[2] = {reinterpret_cast<uint32_t *>(ws + L.keys0),
+                       reinterpret_cast<uint32_t *>(ws + L.keys1)};
+  int32_t *vals[2] = {reinterpret_cast<int32_t *>(ws + L.vals0),
+                      reinterpret_cast<int32_t *>(ws + L.vals1)};
+  uint32_t *hist = reinterpret_cast<uint32_t *>(ws + L.hist);
+  cudaStream_t s = (cudaStream_t)stream;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const int ew_blocks = (int)std::min<long long>((N + kSortThreads - 1) / kSortThreads,
+                                                 (long long)sm_count() * 8);
+  key_kernel<<<ew_blocks, kSortThreads, 0, s>>>(stat, N, keys[0], vals[0], err);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int in = pass & 1, out = in ^ 1;
+    hist_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], N, 8 * pass, hist, L.tiles);
+    scan_kernel<<<1, 1024, 0, s>>>(hist, 256 * L.tiles);
+    scatter_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], vals[in], keys[out], vals[out], N,
+                                                     8 * pass, hist, L.tiles);
+  }
+  GroupStarts gs{};
+  int r = 0;
+  for (int k = K - 1; k >= 0; --k) {
+    gs.start[k] = r;
+    gs.count[k] = counts[k];
+    r += counts[k];
+  }
+  assign_kernel<<<ew_blocks, kSortThreads, 0, s>>>(vals[0], N, K, gs, group_of);
+  return launch_status();
+}
+
+extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const int *budgets,
+                                    int K, int iter, int window_pct, int32_t *idx,
+                                    int32_t *pos, hsa_stream_t stream) {
+  if (!budgets || K < 1) return HSA_ERR_INVALID_ARG;
+  if (K > kMaxGroups) return HSA_ERR_UNSUPPORTED;
+  const int st = hsa_check_budgets(T, budgets, nullptr, K, N);
+  if (st != HSA_OK) return st;
+  const int m = hsa_window_margin(T, window_pct);
+  if (m < 0 || iter < 0 || iter >= T) return HSA_ERR_INVALID_ARG;
+  if (N == 0) return HSA_OK;
+  if (!group_of || !idx) return HSA_ERR_INVALID_ARG;
+  uint32_t mask = 0;
+  for (int k = 0; k < K; ++k) {
+    const bool full = iter < m || iter > T - m - 1;
+    if (full || iter % (T / budgets[k]) == 0) mask |= 1u << k;
+  }
+  // Chunks of at least 4096 tokens, at most one block per SM.
+  const int sms = sm_count();
+  long long chunk = ((long long)N + sms - 1) / sms;
+  chunk = ((chunk + kActThreads - 1) / kActThreads) * kActThreads;
+  if (chunk < 4096) chunk = 4096;
+  const int blocks = (int)(((long long)N + chunk - 1) / chunk);
+  cudaStream_t s = (cudaStream_t)stream;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  if (aligned16(group_of))
+    active_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
+                                                        pos, err);
+  else
+    active_kernel<false><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
+                                                         pos, err);
+  return launch_status();
+}
