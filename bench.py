@@ -1,0 +1,496 @@
+"""Benchmark of the HSA hot path on one GB300 (or N independent replicas).
+
+One step = one pass of the whole hot path over one synthetic HSA layer:
+  partition (once) and then, for each measured iteration i, active set ->
+  gather of the active hidden rows -> KV-cache scatter -> active attention ->
+  cached Euler.
+Default workload: Wan-2.1-1.3B shaped layer, N = 32760 tokens (21x30x52
+grid), 12 heads x 128, bf16, groups 25%@40 + 25%@20 + 50%@10 of T = 40, the
+three iterations i = 0, 2, 1 (100%, 50%, 25% active).
+
+value  = active-attention FLOPs (4 |A| N D H summed over the step) / step
+         time, TFLOP/s, whole job (all replicas); inputs resident in HBM,
+         L2 flushed between steps, CUDA events on the launching stream.
+e2e    = the same metric through the C ABI with host buffers: the step's
+         inputs (statistic, compact Q/K/V and velocities of each iteration's
+         active tokens) are copied from pinned host memory and the attention
+         outputs and the latent are read back inside the timed region.
+--impl reference times the CPU oracle (the reference implementation here) on
+a bounded sample of the same workload, on the host cores.
+
+Multi-GPU: the path is run as independent replicas (one per GPU, no
+collective on the data path); the timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "HSA active-attention TFLOP/s vs BF16 peak; KV-sync/Euler HBM GB/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="hsa", choices=["hsa", "reference"])
+    p.add_argument("--workload", default="wan13b", choices=list(synth.WORKLOADS))
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+# ------------------------------------------------------------ distributed
+
+def dist_setup(backend):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group(backend=backend)
+        return dist, dist.get_rank(), ws, int(os.environ.get("LOCAL_RANK", "0"))
+    return None, 0, 1, 0
+
+
+def max_over_ranks(dist, value: float, device) -> float:
+    if dist is None:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+# ------------------------------------------------------------ peaks/clocks
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples every 200 ms during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, local_rank: int):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        ids = [v.strip() for v in vis.split(",")] if vis else []
+        self.gpu = ids[local_rank] if local_rank < len(ids) else str(local_rank)
+        self.proc = None
+        self.path = os.path.join("/tmp", f"hsa_clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None:
+            return None
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[5:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[3])
+                          if v.lower() == "active"})
+        loaded = [r[0] for r in rows if r[2] > 200.0] or [r[0] for r in rows]
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------- workload
+
+class Layer:
+    """Resident device state and inputs of one HSA layer workload."""
+
+    def __init__(self, w: synth.Workload, dev, rep: int = 0):
+        self.w, self.dev = w, dev
+        N, H, D, C = w.N, w.H, w.D, w.C
+        self.stat_h, self.counts = synth.stat_for(w, rep)
+        seed = lambda t: synth.seed_for(w.cid, rep, t)  # noqa: E731
+        dt = w.dtype
+        self.stat = self.stat_h.to(dev)
+        self.hidden = synth.normal((N, H * D), seed(1), dt).to(dev)
+        self.q = synth.normal((N, H, D), seed(2), dt).to(dev)
+        self.kc = synth.normal((N, H, D), seed(3), dt).to(dev)
+        self.vc = synth.normal((N, H, D), seed(4), dt).to(dev)
+        self.kf = synth.normal((N, H, D), seed(5), dt).to(dev)
+        self.vf = synth.normal((N, H, D), seed(6), dt).to(dev)
+        self.x = synth.normal((N, C), seed(7)).to(dev)
+        self.vh = synth.normal((N, C), seed(8)).to(dev)
+        self.v_fresh = synth.normal((N, C), seed(9)).to(dev)
+        self.group_of = torch.empty(N, dtype=torch.int32, device=dev)
+        self.idx = torch.empty(N, dtype=torch.int32, device=dev)
+        self.pos = torch.empty(N, dtype=torch.int32, device=dev)
+        self.gathered = torch.empty((N, H * D), dtype=self.hidden.dtype, device=dev)
+        self.out = torch.empty((N, H, D), dtype=self.q.dtype, device=dev)
+        self.iters = list(w.iters)
+
+    def bytes_resident(self):
+        return sum(t.numel() * t.element_size() for t in
+                   (self.hidden, self.q, self.kc, self.vc, self.kf, self.vf, self.x, self.vh,
+                    self.v_fresh, self.gathered, self.out))
+
+
+def algorithmic(w, n_act):
+    """Algorithmic FLOPs / bytes per launch of each kernel (see design notes)."""
+    N, H, D, C = w.N, w.H, w.D, w.C
+    eb = 2 if w.dtype == "bf16" else 4
+    row = H * D * eb
+    return {
+        "attention_flops": 4.0 * n_act * N * D * H,
+        "attention_bytes": (2 * n_act + 2 * N) * H * D * eb + 4 * n_act,
+        "gather": n_act * (2 * row + 4),
+        "scatter": n_act * (4 * row + 4),
+        "euler": (N - n_act) * 12 * C + n_act * 16 * C + 4 * N,
+        "active": 4 * N + 4 * n_act + 4 * N,
+    }
+
+
+# ---------------------------------------------------------------- hsa arm
+
+def run_hsa(args, dist, rank, world, local_rank):
+    import paper_2605_06892_gb300 as hsa
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    w = synth.WORKLOADS[args.workload]
+    L = Layer(w, dev)
+    T, budgets = w.T, w.budgets
+    sig = hsa.hsa_sigma_schedule(T, w.shift)
+    ws = torch.empty(hsa.hsa_partition_workspace_bytes(w.N), dtype=torch.uint8, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    n_of = {it: hsa.hsa_active_count(budgets, L.counts, T, it, w.window_pct) for it in L.iters}
+    launches_per_step = 14 + 5 * len(L.iters)
+
+    kinds = ("partition", "active", "gather", "scatter", "attention", "euler")
+
+    def step(record):
+        """One pass of the hot path; record(kind, fn) launches fn between events."""
+        record("partition", lambda: hsa.hsa_partition(L.stat, T, budgets, L.counts, L.group_of,
+                                                      ws, stream))
+        for it in L.iters:
+            n = n_of[it]
+            ds = sig[it + 1] - sig[it]
+            record("active", lambda: hsa.hsa_partition_active(L.group_of, T, budgets, it, L.idx,
+                                                              L.pos, w.window_pct, stream))
+            record("gather", lambda: hsa.hsa_gather_active(L.hidden, L.idx, n, L.gathered,
+                                                           stream))
+            record("scatter", lambda: hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, n,
+                                                              stream))
+            record("attention", lambda: hsa.hsa_active_attention(L.q, L.idx, n, L.kc, L.vc,
+                                                                 L.out, 0.0, stream))
+            record("euler", lambda: hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n,
+                                                         stream))
+
+    plain = lambda kind, fn: fn()  # noqa: E731
+    for _ in range(args.warmup):
+        flush.zero_()
+        step(plain)
+    torch.cuda.synchronize()
+    assert hsa.hsa_get_device_error(stream) == 0
+
+    per_kernel = {k: [] for k in kinds}
+    step_events = []
+
+    def timed(kind, fn):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        per_kernel[kind].append((a, b))
+
+    barrier(dist)
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks:
+        for _ in range(args.steps):
+            flush.zero_()                       # L2 flush, outside the step's events
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record(stream)
+            step(timed)
+            s1.record(stream)
+            step_events.append((s0, s1))
+        torch.cuda.synchronize()
+    barrier(dist)
+    step_ms = [a.elapsed_time(b) for a, b in step_events]
+    total_ms = max_over_ranks(dist, sum(step_ms), dev)
+    ms_per_step = total_ms / args.steps
+    kern_ms = {k: sum(a.elapsed_time(b) for a, b in v) / args.steps for k, v in per_kernel.items()}
+    status = hsa.hsa_get_device_error(stream)
+    assert status == 0, f"device error {status}"
+
+    flops_step = sum(algorithmic(w, n_of[it])["attention_flops"] for it in L.iters)
+    value = world * flops_step / (ms_per_step * 1e-3) / 1e12
+
+    # memory-bound kernels: algorithmic bytes per step / time per step
+    bytes_step = {k: sum(algorithmic(w, n_of[it])[k] for it in L.iters)
+                  for k in ("gather", "scatter", "euler", "active")}
+    peaks, peak_src = load_peaks()
+    kernels = {
+        "attention": {"ms": kern_ms["attention"],
+                      "tflops": flops_step / (kern_ms["attention"] * 1e-3) / 1e12},
+        "partition": {"ms": kern_ms["partition"]},
+    }
+    for k in ("gather", "scatter", "euler", "active"):
+        gbs = bytes_step[k] / (kern_ms[k] * 1e-3) / 1e9
+        kernels[k] = {"ms": kern_ms[k], "gbs": gbs, "frac_hbm": gbs / peaks["hbm_gbs"]}
+    per_iter = {}
+    for it in L.iters:
+        per_iter[str(it)] = {"n_active": n_of[it], "frac": n_of[it] / w.N}
+
+    att_tflops = kernels["attention"]["tflops"]
+    roofline = {"bound": "tensor", "achieved": att_tflops, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": att_tflops / peaks["bf16_tflops"],
+                "traffic": profiled_traffic(w), "peak_source": f"{peak_src} bf16 burst",
+                "frac_sustained": att_tflops / peaks["bf16_tflops_sustained"]}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) Q/K/V, lognormal statistic; no model weights)",
+        "config": {"workload": f"{w.name}: N={w.N} ({w.grid[0]}x{w.grid[1]}x{w.grid[2]}), "
+                               f"H={w.H}, D={w.D}, budgets={list(budgets)}, "
+                               f"counts={list(L.counts)}, T={T}, iterations={L.iters}",
+                   "per_iteration": per_iter, "parallelism": f"replicas x{world}",
+                   "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
+                   "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
+        "kernels": kernels, "roofline": roofline,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks.summary(),
+    }
+    if not args.no_e2e:
+        line["e2e"] = run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, L)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
+    """Same step through the C ABI with host buffers (pinned), copies timed."""
+    w = L.w
+    T, budgets = w.T, w.budgets
+    n_max = max(n_of.values())
+    pin = lambda t: t.cpu().pin_memory()  # noqa: E731
+    h_stat = pin(L.stat)
+    h_q = pin(L.q[:n_max])                      # compact active queries
+    h_kf, h_vf = pin(L.kf[:n_max]), pin(L.vf[:n_max])
+    h_vfr = pin(L.v_fresh[:n_max])
+    h_out = torch.empty((n_max, w.H, w.D), dtype=L.out.dtype).pin_memory()
+    h_x = torch.empty_like(L.x, device="cpu").pin_memory()
+    d_q = torch.empty_like(L.q[:n_max])
+    ws = torch.empty(hsa.hsa_partition_workspace_bytes(w.N), dtype=torch.uint8, device=dev)
+    h2d = L.stat.numel() * 4
+    d2h = h_x.numel() * 4
+    for it in L.iters:
+        n = n_of[it]
+        h2d += n * w.H * w.D * 2 * 3 + n * w.C * 4
+        d2h += n * w.H * w.D * 2
+
+    def step():
+        L.stat.copy_(h_stat, non_blocking=True)
+        hsa.hsa_partition(L.stat, T, budgets, L.counts, L.group_of, ws, stream)
+        for it in L.iters:
+            n = n_of[it]
+            ds = sig[it + 1] - sig[it]
+            d_q[:n].copy_(h_q[:n], non_blocking=True)
+            L.kf[:n].copy_(h_kf[:n], non_blocking=True)
+            L.vf[:n].copy_(h_vf[:n], non_blocking=True)
+            L.v_fresh[:n].copy_(h_vfr[:n], non_blocking=True)
+            hsa.hsa_partition_active(L.group_of, T, budgets, it, L.idx, L.pos, w.window_pct,
+                                     stream)
+            hsa.hsa_gather_active(L.hidden, L.idx, n, L.gathered, stream)
+            hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, n, stream)
+            hsa.hsa_active_attention(d_q, None, n, L.kc, L.vc, L.out, 0.0, stream)
+            h_out[:n].copy_(L.out[:n], non_blocking=True)
+            hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n, stream)
+        h_x.copy_(L.x, non_blocking=True)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(dist)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist)
+    ms = max_over_ranks(dist, a.elapsed_time(b), dev) / args.steps
+    assert hsa.hsa_get_device_error(stream) == 0
+    return {"value": world * flops_step / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+def profiled_traffic(w):
+    """DRAM bytes per attention launch from the committed ncu summary, if it
+    was taken on the current attention source; else None."""
+    path = os.path.join(ROOT, "profiles", f"attention_{w.name}.md")
+    src = os.path.join(ROOT, "paper_2605_06892_gb300", "csrc", "hsa_attention.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        fields = {}
+        for line in open(path):
+            if line.startswith("traffic_per_launch_bytes:") or line.startswith("source_sha256:"):
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+        if fields.get("source_sha256") == sha:
+            return float(fields["traffic_per_launch_bytes"])
+    except (OSError, KeyError, ValueError):
+        pass
+    return None
+
+
+# ----------------------------------------------------------- CPU oracle leg
+
+def _oracle_sample(w, stat, counts, tensors, rows_per_iter, iters):
+    """The oracle's pass over one bounded sample of the workload: partition,
+    active set, gather, scatter and cached Euler at full size, attention for
+    `rows_per_iter` active query rows (all heads, all N keys) per iteration.
+    Returns (seconds, attention FLOPs done)."""
+    import oracle
+    hidden, q, kc, vc, kf, vf, x, vh, vfr = tensors
+    sig = oracle.sigmas(w.T, w.shift)
+    t0 = time.perf_counter()
+    g = oracle.partition(stat, w.T, w.budgets, counts)
+    flops = 0.0
+    for it in iters:
+        idx, pos = oracle.active_set(g, w.T, w.budgets, it, w.window_pct)
+        n = idx.numel()
+        oracle.gather(hidden, idx)
+        oracle.kv_scatter(kc, vc, kf[:n], vf[:n], idx)
+        rows = idx[:rows_per_iter]
+        oracle.attention(q, kc, vc, q_idx=rows)
+        flops += 4.0 * rows.numel() * w.N * w.D * w.H
+        oracle.cached_euler_f32(x, vh, vfr[:n], pos, float(sig[it + 1] - sig[it]))
+    return time.perf_counter() - t0, flops
+
+
+def _host_tensors(w, rep=0):
+    seed = lambda t: synth.seed_for(w.cid, rep, t)  # noqa: E731
+    dt = w.dtype
+    N, H, D, C = w.N, w.H, w.D, w.C
+    return (synth.normal((N, H * D), seed(1), dt), synth.normal((N, H, D), seed(2), dt),
+            synth.normal((N, H, D), seed(3), dt), synth.normal((N, H, D), seed(4), dt),
+            synth.normal((N, H, D), seed(5), dt), synth.normal((N, H, D), seed(6), dt),
+            synth.normal((N, C), seed(7)), synth.normal((N, C), seed(8)),
+            synth.normal((N, C), seed(9)))
+
+
+def cpu_baseline(w, L=None, target_s=15.0):
+    """Oracle timed on the host cores on a bounded sample (single thread)."""
+    stat, counts = synth.stat_for(w)
+    tensors = _host_tensors(w)
+    t1, f1 = _oracle_sample(w, stat, counts, tensors, 1, w.iters[:1])
+    per_row = t1 / max(f1, 1.0)
+    rows = max(1, int(target_s / max(per_row * 4.0 * w.N * w.D * w.H, 1e-9) / len(w.iters)))
+    t, f = _oracle_sample(w, stat, counts, tensors, rows, w.iters)
+    return {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+            "sample": f"partition, active sets, gather, KV scatter and cached Euler at full "
+                      f"size plus attention of {rows} active query rows x {w.H} heads x "
+                      f"{w.N} keys in each of iterations {list(w.iters)}, fp64, "
+                      f"{t:.1f} s single-threaded"}
+
+
+def run_reference(args, dist, rank, world):
+    """The oracle as the reference arm: each step is a bounded sample of the
+    workload (4 query rows per iteration), timed on the host cores."""
+    if rank != 0:
+        return
+    w = synth.WORKLOADS[args.workload]
+    stat, counts = synth.stat_for(w)
+    tensors = _host_tensors(w)
+    rows = 4
+    for _ in range(args.warmup):
+        _oracle_sample(w, stat, counts, tensors, rows, w.iters)
+    tot_t, tot_f = 0.0, 0.0
+    for _ in range(args.steps):
+        t, f = _oracle_sample(w, stat, counts, tensors, rows, w.iters)
+        tot_t += t
+        tot_f += f
+    value = tot_f / tot_t / 1e12
+    sample = (f"oracle pass per step: full-size partition/active set/gather/scatter/Euler and "
+              f"attention of {rows} query rows x {w.H} heads per iteration {list(w.iters)}")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * tot_t / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{w.name}: N={w.N}, H={w.H}, D={w.D}"},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        dist, rank, world, _ = dist_setup("gloo")
+        run_reference(args, dist, rank, world)
+        return
+    dist, rank, world, local_rank = dist_setup("nccl")
+    run_hsa(args, dist, rank, world, local_rank)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

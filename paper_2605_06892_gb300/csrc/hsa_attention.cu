@@ -170,6 +170,32 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
       : "memory");
 }
 
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+      "%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -214,6 +240,81 @@ struct TcArgs {
   int n_active, N, H, q_rows, n_kv_tiles;
   float scale_log2;
 };
+
+// Scores of one 128-key tile for this thread's row: S from TMEM (one read),
+// the running maximum (moved only when it grows by more than 2^8, with O
+// rescaled in TMEM), P = 2^(s*scale*log2e - m) as bf16 pairs written over the
+// first 64 S columns, and the running sum.  kTail masks keys >= valid (the
+// last, ragged tile); full tiles take no per-key test.  Reductions use eight
+// independent partial results to keep dependency chains short.
+template <int D, bool kTail>
+__device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid, bool first,
+                                             float sl2, float &m_run, float &l_run) {
+  uint32_t r[128];
+  tmem_ld32(tS, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
+  tmem_ld32(tS + 32, *reinterpret_cast<uint32_t(*)[32]>(&r[32]));
+  tmem_ld32(tS + 64, *reinterpret_cast<uint32_t(*)[32]>(&r[64]));
+  tmem_ld32(tS + 96, *reinterpret_cast<uint32_t(*)[32]>(&r[96]));
+  tmem_wait_ld();
+  if (kTail) {
+#pragma unroll
+    for (int i = 0; i < 128; ++i)
+      if (i >= valid) r[i] = __float_as_uint(-INFINITY);
+  }
+  float pm[8];
+#pragma unroll
+  for (int p = 0; p < 8; ++p) {
+    float m = __uint_as_float(r[16 * p]);
+#pragma unroll
+    for (int i = 1; i < 16; i += 2)
+      m = max3f(m, __uint_as_float(r[16 * p + i]), __uint_as_float(r[16 * p + i + 1]));
+    m = fmaxf(m, __uint_as_float(r[16 * p + 15]));
+    pm[p] = m;
+  }
+  const float mx = fmaxf(max3f(pm[0], pm[1], pm[2]),
+                         fmaxf(max3f(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+  const float m_new = fmaxf(m_run, mx * sl2);
+  if (first) {
+    m_run = m_new;
+  } else {
+    const bool need = m_new > m_run + kRescaleLog2;
+    if (__any_sync(0xffffffffu, need)) {
+      const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
+      if (need) {
+        l_run *= alpha;
+        m_run = m_new;
+      }
+#pragma unroll
+      for (int c = 0; c < D / 16; ++c) {
+        uint32_t o[16];
+        tmem_ld16(tO + 16 * c, o);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+        tmem_st16(tO + 16 * c, o);
+      }
+      tmem_wait_st();
+    }
+  }
+  const float neg_m = -m_run;
+  float ps[8];
+#pragma unroll
+  for (int p = 0; p < 8; ++p) ps[p] = 0.f;
+  // All 128 scores are in registers, so P may overwrite S column by column.
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint32_t pk[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const float p0 = fast_exp2(fmaf(__uint_as_float(r[64 * h + 2 * i]), sl2, neg_m));
+      const float p1 = fast_exp2(fmaf(__uint_as_float(r[64 * h + 2 * i + 1]), sl2, neg_m));
+      ps[i & 7] += p0 + p1;
+      pk[i] = pack_bf16(p0, p1);
+    }
+    tmem_st32(tS + 32 * h, pk);
+  }
+  l_run += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+}
 
 template <int D>
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -386,69 +487,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       if (!(ok = mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err))) break;
       fence_after();
       const int valid = a.N - j * kBN;             // keys of this tile that exist
-      // Pass 1: row maximum over the 128 scores, 64 columns per TMEM read.
-      float mx = -INFINITY;
-#pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2) {
-        uint32_t raw[2][32];
-        tmem_ld32(tS + 64 * h2, raw[0]);
-        tmem_ld32(tS + 64 * h2 + 32, raw[1]);
-        tmem_wait_ld();
-#pragma unroll
-        for (int c = 0; c < 2; ++c)
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float v = __uint_as_float(raw[c][i]);
-            mx = (64 * h2 + 32 * c + i < valid) ? fmaxf(mx, v) : mx;
-          }
-      }
-      const float m_new = fmaxf(m_run, mx * sl2);
-      if (j == 0) {
-        m_run = m_new;
-      } else {
-        const bool need = m_new > m_run + kRescaleLog2;
-        if (__any_sync(0xffffffffu, need)) {
-          const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
-          if (need) {
-            l_run *= alpha;
-            m_run = m_new;
-          }
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(tO + 32 * c, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-            tmem_st32(tO + 32 * c, o);
-          }
-          tmem_wait_st();
-        }
-      }
-      // Pass 2: p = 2^(s*scale*log2e - m), packed to bf16 pairs into the first
-      // 64 columns of S.  The 64 scores of half h2 are read before the P
-      // columns [32*h2, 32*h2+32) they overlap are written.
-      float rs = 0.f;
-#pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2) {
-        uint32_t raw[2][32];
-        tmem_ld32(tS + 64 * h2, raw[0]);
-        tmem_ld32(tS + 64 * h2 + 32, raw[1]);
-        tmem_wait_ld();
-        uint32_t pk[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int col = 64 * h2 + 2 * i;
-          const float s0 = __uint_as_float(raw[(2 * i) / 32][(2 * i) % 32]);
-          const float s1 = __uint_as_float(raw[(2 * i + 1) / 32][(2 * i + 1) % 32]);
-          const float p0 = col < valid ? fast_exp2(fmaf(s0, sl2, -m_run)) : 0.f;
-          const float p1 = col + 1 < valid ? fast_exp2(fmaf(s1, sl2, -m_run)) : 0.f;
-          rs += p0 + p1;
-          pk[i] = pack_bf16(p0, p1);
-        }
-        tmem_st32(tS + 32 * h2, pk);
-      }
-      l_run += rs;
+      if (valid >= kBN)
+        softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
+      else
+        softmax_tile<D, true>(tS, tO, valid, j == 0, sl2, m_run, l_run);
       tmem_wait_st();
       fence_before();
       mbar_arrive(&bar_p[t]);

@@ -57,7 +57,7 @@ __device__ __forceinline__ void copy_rows(long long n_rows, int vecs, int lpr_lo
 }
 
 __global__ void __launch_bounds__(kThreads)
-gather_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
+gather_rows_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
               const int32_t *__restrict__ idx, int n_active, int N, int vecs,
               int lpr_log2, unsigned *err) {
   copy_rows(n_active, vecs, lpr_log2, [&](long long j, const uint4 *&s, uint4 *&d) {
@@ -75,7 +75,7 @@ gather_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
 // Rows 0..n_active-1 are K rows, n_active..2*n_active-1 the V rows, so a warp
 // moves K and V rows of different tokens with the same code.
 __global__ void __launch_bounds__(kThreads)
-scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
+kv_scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
                const uint4 *__restrict__ kf, const uint4 *__restrict__ vf,
                const int32_t *__restrict__ idx, int n_active, int N, int vecs,
                int lpr_log2, unsigned *err) {
@@ -96,7 +96,7 @@ scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
 // x[n] = fma(vhat[n], dsigma, x[n]) with vhat[n] refreshed from
 // v_fresh[pos[n]] when pos[n] >= 0.  A row is C/4 float4 vectors.
 __global__ void __launch_bounds__(kThreads)
-euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
+cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
              const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
              int N, int vecs, int lpr_log2, float dsigma, int n_fresh_rows, unsigned *err) {
   const int L = 1 << lpr_log2;
@@ -174,7 +174,7 @@ extern "C" int hsa_gather_active(const void *src, size_t row_bytes, int N,
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   const int L = lanes_per_row(vecs);
-  gather_kernel<<<grid_for(n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
+  gather_rows_kernel<<<grid_for(n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
       (const uint4 *)src, (uint4 *)dst, idx, n_active, N, (int)vecs, log2i(L), err);
   return launch_status();
 }
@@ -196,7 +196,7 @@ extern "C" int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_f
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   const int L = lanes_per_row(vecs);
-  scatter_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
+  kv_scatter_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
       (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
       n_active, N, (int)vecs, log2i(L), err);
   return launch_status();
@@ -214,7 +214,7 @@ extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
   if (!err) return HSA_ERR_CUDA;
   const int vecs = C / 4;
   const int L = lanes_per_row(vecs);
-  euler_kernel<<<grid_for(N, L), kThreads, 0, (cudaStream_t)stream>>>(
+  cached_euler_kernel<<<grid_for(N, L), kThreads, 0, (cudaStream_t)stream>>>(
       (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, N, vecs, log2i(L), dsigma,
       pos ? n_fresh : 0, err);
   return launch_status();

@@ -54,7 +54,7 @@ SortLayout sort_layout(int N) {
 }
 
 __global__ void __launch_bounds__(kSortThreads)
-key_kernel(const float *__restrict__ stat, int N, uint32_t *__restrict__ keys,
+radix_key_kernel(const float *__restrict__ stat, int N, uint32_t *__restrict__ keys,
            int32_t *__restrict__ vals, unsigned *err) {
   for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < N; n += gridDim.x * blockDim.x) {
     const float f = stat[n];
@@ -67,7 +67,7 @@ key_kernel(const float *__restrict__ stat, int N, uint32_t *__restrict__ keys,
 }
 
 __global__ void __launch_bounds__(kSortThreads)
-hist_kernel(const uint32_t *__restrict__ keys, int N, int shift, uint32_t *__restrict__ hist,
+radix_hist_kernel(const uint32_t *__restrict__ keys, int N, int shift, uint32_t *__restrict__ hist,
             int tiles) {
   __shared__ uint32_t h[256];
   h[threadIdx.x] = 0;
@@ -84,7 +84,7 @@ hist_kernel(const uint32_t *__restrict__ keys, int N, int shift, uint32_t *__res
 
 // Exclusive scan, in place, of the 256*tiles counts in digit-major order, by
 // one block of 1024 threads, each owning a contiguous run.
-__global__ void __launch_bounds__(1024) scan_kernel(uint32_t *__restrict__ hist, int total) {
+__global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t *__restrict__ hist, int total) {
   __shared__ uint32_t warp_sum[32];
   const int per = (total + 1023) / 1024;
   const int b = threadIdx.x * per;
@@ -124,7 +124,7 @@ __global__ void __launch_bounds__(1024) scan_kernel(uint32_t *__restrict__ hist,
 // the tile is (earlier warps' count) + (this warp's running count) + (earlier
 // lanes of this step).
 __global__ void __launch_bounds__(kSortThreads)
-scatter_kernel(const uint32_t *__restrict__ kin, const int32_t *__restrict__ vin,
+radix_scatter_kernel(const uint32_t *__restrict__ kin, const int32_t *__restrict__ vin,
                uint32_t *__restrict__ kout, int32_t *__restrict__ vout, int N, int shift,
                const uint32_t *__restrict__ offsets, int tiles) {
   __shared__ uint32_t cnt[kWarps][256];
@@ -175,7 +175,7 @@ scatter_kernel(const uint32_t *__restrict__ kin, const int32_t *__restrict__ vin
 }
 
 __global__ void __launch_bounds__(kSortThreads)
-assign_kernel(const int32_t *__restrict__ sorted_tokens, int N, int K, GroupStarts gs,
+group_assign_kernel(const int32_t *__restrict__ sorted_tokens, int N, int K, GroupStarts gs,
               int32_t *__restrict__ group_of) {
   for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < N; r += gridDim.x * blockDim.x) {
     int g = 0;
@@ -191,7 +191,7 @@ constexpr int kActThreads = 1024;
 
 template <bool kVec>
 __global__ void __launch_bounds__(kActThreads)
-active_kernel(const int32_t *__restrict__ group_of, int N, int K, uint32_t mask, int chunk,
+active_set_kernel(const int32_t *__restrict__ group_of, int N, int K, uint32_t mask, int chunk,
               int32_t *__restrict__ idx, int32_t *__restrict__ pos, unsigned *err) {
   __shared__ int warp_cnt[32];
   __shared__ int block_base;
@@ -284,12 +284,12 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
   if (!err) return HSA_ERR_CUDA;
   const int ew_blocks = (int)std::min<long long>((N + kSortThreads - 1) / kSortThreads,
                                                  (long long)sm_count() * 8);
-  key_kernel<<<ew_blocks, kSortThreads, 0, s>>>(stat, N, keys[0], vals[0], err);
+  radix_key_kernel<<<ew_blocks, kSortThreads, 0, s>>>(stat, N, keys[0], vals[0], err);
   for (int pass = 0; pass < 4; ++pass) {
     const int in = pass & 1, out = in ^ 1;
-    hist_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], N, 8 * pass, hist, L.tiles);
-    scan_kernel<<<1, 1024, 0, s>>>(hist, 256 * L.tiles);
-    scatter_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], vals[in], keys[out], vals[out], N,
+    radix_hist_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], N, 8 * pass, hist, L.tiles);
+    radix_scan_kernel<<<1, 1024, 0, s>>>(hist, 256 * L.tiles);
+    radix_scatter_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], vals[in], keys[out], vals[out], N,
                                                      8 * pass, hist, L.tiles);
   }
   GroupStarts gs{};
@@ -299,7 +299,7 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
     gs.count[k] = counts[k];
     r += counts[k];
   }
-  assign_kernel<<<ew_blocks, kSortThreads, 0, s>>>(vals[0], N, K, gs, group_of);
+  group_assign_kernel<<<ew_blocks, kSortThreads, 0, s>>>(vals[0], N, K, gs, group_of);
   return launch_status();
 }
 
@@ -329,10 +329,10 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   if (aligned16(group_of))
-    active_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
+    active_set_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
                                                         pos, err);
   else
-    active_kernel<false><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
+    active_set_kernel<false><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
                                                          pos, err);
   return launch_status();
 }
