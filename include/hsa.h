@@ -118,6 +118,30 @@ int hsa_partition(const float *stat, int N, int T, const int *budgets,
                   const int *counts, int K, int32_t *group_of, void *workspace,
                   size_t workspace_bytes, hsa_stream_t stream);
 
+/* Largest N accepted by hsa_partition_static. */
+#define HSA_PARTITION_STATIC_MAX_TOKENS 262144
+
+/* hsa_partition without a workspace argument, for callers that cannot
+ * allocate device memory for one: a plugin inside a host framework that owns
+ * all device memory and offers it no allocator, or a latency-critical loop
+ * that must not call cudaMalloc/cudaFree (they may synchronise the device).
+ * The paper has no counterpart; the ranking and group assignment are exactly
+ * those of hsa_partition (same arguments, same results).
+ * Scratch: a fixed device array inside the library, about 4.3 MB, sized for
+ * N <= HSA_PARTITION_STATIC_MAX_TOKENS; every GPU that loads the library
+ * holds it until the process exits.  Larger N returns HSA_ERR_UNSUPPORTED
+ * before any launch.  Nothing is allocated: no cudaMalloc, cudaFree or
+ * allocating library call is made.
+ * The first call on a device looks up the array's device address (a CUDA
+ * runtime query) for that device, so make that first call before any stream
+ * capture.  Every call on a device shares the one array and finds the last
+ * call's contents there (none need to start at zero); calls whose work
+ * overlaps on the GPU (other streams, or other host threads) race on it and
+ * must be serialised by the caller. */
+int hsa_partition_static(const float *stat, int N, int T, const int *budgets,
+                         const int *counts, int K, int32_t *group_of,
+                         hsa_stream_t stream);
+
 /* ---------------------------------------------------- a2 active set per step */
 
 /* Active set A_i (Sec. 2.3; Fig. 1): token n is active at iteration iter iff

@@ -20,7 +20,7 @@ __all__ = [
     "HsaError", "lib", "library_path", "HSA_BF16", "HSA_F32",
     "hsa_status_string", "hsa_version", "hsa_check_budgets", "hsa_window_margin",
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
-    "hsa_partition", "hsa_partition_active", "hsa_gather_active",
+    "hsa_partition", "hsa_partition_static", "hsa_partition_active", "hsa_gather_active",
     "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_cached_euler",
     "hsa_get_device_error",
 ]
@@ -29,6 +29,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 library_path = os.path.join(_HERE, "libhsa.so")
 
 HSA_BF16, HSA_F32 = 0, 1
+HSA_PARTITION_STATIC_MAX_TOKENS = 262144
 STATUS = {0: "HSA_OK", -1: "HSA_ERR_INVALID_ARG", -2: "HSA_ERR_NOT_DIVISOR",
           -3: "HSA_ERR_BAD_COUNTS", -4: "HSA_ERR_UNSUPPORTED", -5: "HSA_ERR_NONFINITE",
           -6: "HSA_ERR_INDEX", -7: "HSA_ERR_TIMEOUT", -8: "HSA_ERR_CUDA",
@@ -53,6 +54,7 @@ _SIGS = {
     "hsa_partition_workspace_bytes": ([_c_int], _c_sz),
     "hsa_partition": ([_c_p, _c_int, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p, _c_sz, _c_p],
                       _c_int),
+    "hsa_partition_static": ([_c_p, _c_int, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p], _c_int),
     "hsa_partition_active": ([_c_p, _c_int, _c_int, _c_p, _c_int, _c_int, _c_int, _c_p, _c_p,
                               _c_p], _c_int),
     "hsa_gather_active": ([_c_p, _c_sz, _c_int, _c_p, _c_int, _c_p, _c_p], _c_int),
@@ -166,6 +168,15 @@ def hsa_partition(stat, T: int, budgets, counts, group_of, workspace, stream=Non
     _check(lib().hsa_partition(_p(stat), N, T, _host_ints(budgets), _host_ints(counts),
                                len(budgets), _p(group_of), _p(workspace), ws_bytes,
                                _stream(stream)), "hsa_partition")
+
+
+def hsa_partition_static(stat, T: int, budgets, counts, group_of, stream=None) -> None:
+    """hsa_partition with the library's own fixed scratch instead of a caller
+    workspace (N <= HSA_PARTITION_STATIC_MAX_TOKENS); calls must not overlap
+    on the GPU."""
+    _check(lib().hsa_partition_static(_p(stat), stat.numel(), T, _host_ints(budgets),
+                                      _host_ints(counts), len(budgets), _p(group_of),
+                                      _stream(stream)), "hsa_partition_static")
 
 
 def hsa_partition_active(group_of, T: int, budgets, iter_: int, idx, pos=None,

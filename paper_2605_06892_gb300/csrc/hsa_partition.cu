@@ -15,6 +15,7 @@
 // is cheap at the token counts of a video DiT), then compacts its own chunk
 // with warp ballots and a block scan.
 #include <algorithm>
+#include <atomic>
 
 #include "hsa_internal.cuh"
 
@@ -335,4 +336,54 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
     active_set_kernel<false><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
                                                          pos, err);
   return launch_status();
+}
+
+// ----------------------------------------------- partition without allocation
+//
+// Variant of hsa_partition for callers that cannot hand the library a
+// workspace: a plugin running inside a host framework that owns all device
+// memory and exposes no allocator to it, or a latency-critical loop where
+// cudaMalloc/cudaFree (which may synchronise the device) are not acceptable.
+// Its scratch is a fixed file-scope device array sized for
+// HSA_PARTITION_STATIC_MAX_TOKENS tokens; every GPU that loads the library
+// holds it until the process exits.
+
+namespace {
+
+constexpr size_t static_workspace_bytes(size_t n) {
+  return 4 * ((n * 4 + 255) / 256 * 256) + ((256 * ((n + kTile - 1) / kTile) * 4 + 255) / 256 * 256);
+}
+
+constexpr size_t kStaticScratchBytes = static_workspace_bytes(HSA_PARTITION_STATIC_MAX_TOKENS);
+
+// The host cannot use this symbol as a device address; the set-up below asks
+// the runtime for the device address once per device.
+static __device__ __align__(256) unsigned char g_partition_scratch[kStaticScratchBytes];
+
+std::atomic<void *> g_scratch_ptr[64];
+
+// Device address of g_partition_scratch on the current device (nullptr on
+// failure).  The first call on a device resolves it.
+void *static_scratch() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  void *p = g_scratch_ptr[dev].load(std::memory_order_acquire);
+  if (!p) {
+    if (cudaGetSymbolAddress(&p, g_partition_scratch) != cudaSuccess || !p) return nullptr;
+    g_scratch_ptr[dev].store(p, std::memory_order_release);
+  }
+  return p;
+}
+
+}  // namespace
+
+extern "C" int hsa_partition_static(const float *stat, int N, int T, const int *budgets,
+                                    const int *counts, int K, int32_t *group_of,
+                                    hsa_stream_t stream) {
+  if (N > HSA_PARTITION_STATIC_MAX_TOKENS) return HSA_ERR_UNSUPPORTED;
+  if (N >= 0 && hsa_partition_workspace_bytes(N) > kStaticScratchBytes) return HSA_ERR_UNSUPPORTED;
+  void *scratch = static_scratch();
+  if (!scratch) return HSA_ERR_CUDA;
+  return hsa_partition(stat, N, T, budgets, counts, K, group_of, scratch, kStaticScratchBytes,
+                       stream);
 }
