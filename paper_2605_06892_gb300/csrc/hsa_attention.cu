@@ -8,7 +8,8 @@
 //               into a ring of shared-memory slots (rows >= N are zero-filled).
 //   warp 1      tensor-core issuer (one thread): S_t = Q_t K^T into TMEM and
 //               O_t += P_t V from TMEM P and shared V, tcgen05.mma kind::f16.
-//   warps 2-5   softmax of Q tile 0, warps 6-9 softmax of Q tile 1: each
+//   warps 2-3   idle (they complete the first warpgroup).
+//   warps 4-7   softmax of Q tile 0, warps 8-11 softmax of Q tile 1: each
 //               thread owns one query row (its TMEM lane; a warp may only
 //               reach the lane quarter warp%4), reads its S row,
 //               keeps the running maximum and sum, writes P as bf16 back into
@@ -19,6 +20,9 @@
 // (and O rescaled in TMEM) when it grows by more than 2^8, so most iterations
 // skip the rescale; the final division by the running sum makes the result
 // exact whatever maximum was used.
+// Registers: the block launches at 168 per thread; the first warpgroup then
+// gives registers back (setmaxnreg.dec to 88) and the two softmax warpgroups
+// take them (setmaxnreg.inc to 208): 128*88 + 256*208 = 384*168.
 // Every mbarrier wait is bounded in time; on a timeout the kernel records
 // HSA_ERR_TIMEOUT, stops issuing work, drains its own copies and MMAs, frees
 // TMEM and returns.
@@ -68,6 +72,20 @@ __device__ __forceinline__ bool mbar_test(uint64_t *b, uint32_t parity) {
   return ok != 0;
 }
 
+// try_wait that lets the hardware suspend the thread for up to ~0.5 ms while
+// the phase is incomplete, so waiting warps take no issue slots from the
+// working ones.
+__device__ __forceinline__ bool mbar_test_suspend(uint64_t *b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(b)), "r"(parity), "r"(500000u)
+      : "memory");
+  return ok != 0;
+}
+
 // About one second at the GB300 clock.
 constexpr long long kWaitCycles = 2000000000LL;
 
@@ -79,7 +97,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile
   if (mbar_test(b, parity)) return true;
   const long long t0 = clock64();
   while (true) {
-    if (mbar_test(b, parity)) return true;
+    if (mbar_test_suspend(b, parity)) return true;
     if (honor_abort && *abort_flag) return false;
     if (clock64() - t0 > kWaitCycles) {
       set_error(err, kErrTimeout);
@@ -190,6 +208,23 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
       : "memory");
 }
 
+// Packed fp32 pairs (sm_100 family): two lanes of work per instruction.
+__device__ __forceinline__ uint64_t pack2(uint32_t lo, uint32_t hi) {
+  return (uint64_t)lo | ((uint64_t)hi << 32);
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float lo_f(uint64_t v) { return __uint_as_float((uint32_t)v); }
+__device__ __forceinline__ float hi_f(uint64_t v) { return __uint_as_float((uint32_t)(v >> 32)); }
+
 __device__ __forceinline__ float max3f(float a, float b, float c) {
   float r;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
@@ -201,6 +236,10 @@ __device__ __forceinline__ void tmem_wait_ld() {
 }
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void named_barrier_sync(int id, int threads) {
+  asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
 __device__ __forceinline__ float fast_exp2(float x) {
@@ -219,7 +258,12 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 constexpr int kBM = 128;         // query rows per Q tile (= TMEM lanes)
 constexpr int kQT = 2;           // Q tiles per CTA
 constexpr int kBN = 128;         // keys per K/V tile
-constexpr int kTcThreads = 320;  // 10 warps
+constexpr int kTcThreads = 384;  // 12 warps = 3 warpgroups
+constexpr int kLaunchRegs = 168;         // registers per thread at launch
+constexpr int kRegsLow = 88;             // producer / MMA warpgroup
+constexpr int kRegsHigh = 208;           // softmax warpgroups
+static_assert(128 * kRegsLow + 256 * kRegsHigh <= kTcThreads * kLaunchRegs,
+              "register split exceeds the launch allocation");
 constexpr int kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.0f;   // lazy rescale threshold, log2 units
 
@@ -274,46 +318,47 @@ __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid
   const float mx = fmaxf(max3f(pm[0], pm[1], pm[2]),
                          fmaxf(max3f(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])));
   const float m_new = fmaxf(m_run, mx * sl2);
-  if (first) {
+  // The reference maximum moves only on the first tile or when it grows by
+  // more than 2^kRescaleLog2; then O (in TMEM) and the sum take the factor
+  // alpha.  O is rescaled after P is written, when the scores are dead.
+  const bool need = first || m_new > m_run + kRescaleLog2;
+  const float alpha = (need && !first) ? fast_exp2(m_run - m_new) : 1.f;
+  if (need) {
+    l_run *= alpha;
     m_run = m_new;
-  } else {
-    const bool need = m_new > m_run + kRescaleLog2;
-    if (__any_sync(0xffffffffu, need)) {
-      const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
-      if (need) {
-        l_run *= alpha;
-        m_run = m_new;
-      }
-#pragma unroll
-      for (int c = 0; c < D / 16; ++c) {
-        uint32_t o[16];
-        tmem_ld16(tO + 16 * c, o);
-        tmem_wait_ld();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-        tmem_st16(tO + 16 * c, o);
-      }
-      tmem_wait_st();
-    }
   }
-  const float neg_m = -m_run;
-  float ps[8];
-#pragma unroll
-  for (int p = 0; p < 8; ++p) ps[p] = 0.f;
+  // x = s*scale*log2e - m for a pair of scores in one packed FMA; p = 2^x.
+  const uint64_t scale2 = pack2(__float_as_uint(sl2), __float_as_uint(sl2));
+  const uint64_t negm2 = pack2(__float_as_uint(-m_run), __float_as_uint(-m_run));
+  uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
   // All 128 scores are in registers, so P may overwrite S column by column.
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     uint32_t pk[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
-      const float p0 = fast_exp2(fmaf(__uint_as_float(r[64 * h + 2 * i]), sl2, neg_m));
-      const float p1 = fast_exp2(fmaf(__uint_as_float(r[64 * h + 2 * i + 1]), sl2, neg_m));
-      ps[i & 7] += p0 + p1;
+      const uint64_t x = fma2(pack2(r[64 * h + 2 * i], r[64 * h + 2 * i + 1]), scale2, negm2);
+      const float p0 = fast_exp2(lo_f(x));
+      const float p1 = fast_exp2(hi_f(x));
+      ps[i & 3] = add2(ps[i & 3], pack2(__float_as_uint(p0), __float_as_uint(p1)));
       pk[i] = pack_bf16(p0, p1);
     }
     tmem_st32(tS + 32 * h, pk);
   }
-  l_run += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+  const uint64_t s01 = add2(ps[0], ps[1]), s23 = add2(ps[2], ps[3]);
+  const uint64_t st = add2(s01, s23);
+  l_run += lo_f(st) + hi_f(st);
+  if (!first && __any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t o[32];
+      tmem_ld32(tO + 32 * c, o);
+      tmem_wait_ld();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+      tmem_st32(tO + 32 * c, o);
+    }
+  }
 }
 
 template <int D>
@@ -385,96 +430,117 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   fence_after();
   const uint32_t tmem = tmem_base_sh;
 
-  if (warp == 0) {
-    // ------------------------------------------------ TMA producer
-    if (lane == 0) {
-      int issued = 0;
-      for (int L = 0; L < 2 * nT; ++L) {
-        const int slot = L % C::kStages, use = L / C::kStages;
-        if (use > 0 && !mbar_wait(&bar_empty[slot], (use - 1) & 1, &abort_flag, a.err)) break;
-        mbar_expect_tx(&bar_full[slot], C::kTileBytes);
-        const CUtensorMap *map = (L & 1) ? &tm_v : &tm_k;
-        uint8_t *dst = sKV + slot * C::kTileBytes;
+  // The warpgroups' code paths never rejoin below: each ends with its own
+  // teardown on named barrier 1, so each path is compiled for its own
+  // register budget.
+  if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
+    if (warp == 0) {
+      // ------------------------------------------------ TMA producer
+      if (lane == 0) {
+        int issued = 0;
+        for (int L = 0; L < 2 * nT; ++L) {
+          const int slot = L % C::kStages, use = L / C::kStages;
+          if (use > 0 && !mbar_wait(&bar_empty[slot], (use - 1) & 1, &abort_flag, a.err)) break;
+          mbar_expect_tx(&bar_full[slot], C::kTileBytes);
+          const CUtensorMap *map = (L & 1) ? &tm_v : &tm_k;
+          uint8_t *dst = sKV + slot * C::kTileBytes;
 #pragma unroll
-        for (int c = 0; c < C::kChunks; ++c)
-          tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, (L >> 1) * kBN);
-        issued = L + 1;
-      }
-      // Drain: every issued copy has landed before the CTA may exit.
-      for (int L = issued > C::kStages ? issued - C::kStages : 0; L < issued; ++L)
-        mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err, false);
-    }
-    __syncwarp();
-  } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t kIdS = idesc_bf16(kBM, kBN, 0);
-      constexpr uint32_t kIdO = idesc_bf16(kBM, D, 1);
-      const uint32_t q_base = smem_addr(sQ);
-      const uint32_t kv_base = smem_addr(sKV);
-      auto slot_addr = [&](int L) { return kv_base + (L % C::kStages) * C::kTileBytes; };
-      auto wait_full = [&](int L) {
-        return mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err);
-      };
-      // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
-      auto issue_s = [&](int t, int L) {
-        const uint32_t qa = q_base + t * C::kTileBytes, ka = slot_addr(L);
-#pragma unroll
-        for (int k = 0; k < D / 16; ++k) {
-          const uint32_t off = (k >> 2) * (kBM * 128) + (k & 3) * 32;
-          mma_ss(tmem + 128 * t, sdesc(qa + off, 16, 1024), sdesc(ka + off, 16, 1024), kIdS,
-                 k > 0);
+          for (int c = 0; c < C::kChunks; ++c)
+            tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, (L >> 1) * kBN);
+          issued = L + 1;
         }
-      };
-      // O_t += P_t V: P in TMEM (bf16 pairs in the S_t columns), V MN-major.
-      auto issue_o = [&](int t, int L, bool acc) {
-        const uint32_t va = slot_addr(L);
-#pragma unroll
-        for (int k = 0; k < kBN / 16; ++k)
-          mma_ts(tmem + C::kOCol0 + D * t, tmem + 128 * t + 8 * k,
-                 sdesc(va + k * 2048, kBN * 128, 1024), kIdO, (acc || k > 0) ? 1u : 0u);
-      };
-      bool ok = wait_full(0);
-      if (ok) {
-        fence_after();
-        issue_s(0, 0);
-        mma_commit(&bar_s[0]);
-        issue_s(1, 0);
-        mma_commit(&bar_s[1]);
-        mma_commit(&bar_empty[0]);
+        // Drain: every issued copy has landed before the CTA may exit.
+        for (int L = issued > C::kStages ? issued - C::kStages : 0; L < issued; ++L)
+          mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err, false);
       }
-      for (int j = 0; ok && j < nT; ++j) {
-        const int Lv = 2 * j + 1, Lk = 2 * j + 2;
-        const bool more = j + 1 < nT;
-        if (!(ok = wait_full(Lv))) break;
-        if (!(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err))) break;
-        fence_after();
-        issue_o(0, Lv, j > 0);
-        if (more) {
-          if (!(ok = wait_full(Lk))) break;
+      __syncwarp();
+      } else if (warp == 1) {
+      // ------------------------------------------------ MMA issuer
+      if (lane == 0) {
+        constexpr uint32_t kIdS = idesc_bf16(kBM, kBN, 0);
+        constexpr uint32_t kIdO = idesc_bf16(kBM, D, 1);
+        const uint32_t q_base = smem_addr(sQ);
+        const uint32_t kv_base = smem_addr(sKV);
+        auto wait_full = [&](int L) {
+          return mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err);
+        };
+        // Descriptors differ only in their start-address field (bits 0-13,
+        // address >> 4), so each MMA adds a constant to a base descriptor.
+        const uint64_t dq0 = sdesc(q_base, 16, 1024);
+        const uint64_t dk0 = sdesc(kv_base, 16, 1024);
+        const uint64_t dv0 = sdesc(kv_base, kBN * 128, 1024);
+        constexpr uint32_t kTile16 = C::kTileBytes >> 4;
+        // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
+        auto issue_s = [&](int t, int L) {
+          const uint64_t dq = dq0 + t * kTile16;
+          const uint64_t dk = dk0 + (L % C::kStages) * kTile16;
+          const uint32_t ts = tmem + 128 * t;
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {
+            const uint32_t off = ((k >> 2) * (kBM * 128) + (k & 3) * 32) >> 4;
+            mma_ss(ts, dq + off, dk + off, kIdS, k > 0);
+          }
+        };
+        // O_t += P_t V: P in TMEM (bf16 pairs in the S_t columns), V MN-major.
+        auto issue_o = [&](int t, int L, bool acc) {
+          const uint64_t dv = dv0 + (L % C::kStages) * kTile16;
+          const uint32_t to = tmem + C::kOCol0 + D * t, tp = tmem + 128 * t;
+#pragma unroll
+          for (int k = 0; k < kBN / 16; ++k)
+            mma_ts(to, tp + 8 * k, dv + ((k * 2048) >> 4), kIdO, (acc || k > 0) ? 1u : 0u);
+        };
+        bool ok = wait_full(0);
+        if (ok) {
           fence_after();
-          issue_s(0, Lk);
+          issue_s(0, 0);
           mma_commit(&bar_s[0]);
-        }
-        if (!(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err))) break;
-        fence_after();
-        issue_o(1, Lv, j > 0);
-        mma_commit(&bar_empty[Lv % C::kStages]);
-        if (more) {
-          issue_s(1, Lk);
+          issue_s(1, 0);
           mma_commit(&bar_s[1]);
-          mma_commit(&bar_empty[Lk % C::kStages]);
+          mma_commit(&bar_empty[0]);
         }
+        for (int j = 0; ok && j < nT; ++j) {
+          const int Lv = 2 * j + 1, Lk = 2 * j + 2;
+          const bool more = j + 1 < nT;
+          if (!(ok = wait_full(Lv))) break;
+          if (!(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err))) break;
+          fence_after();
+          issue_o(0, Lv, j > 0);
+          if (more) {
+            if (!(ok = wait_full(Lk))) break;
+            fence_after();
+            issue_s(0, Lk);
+            mma_commit(&bar_s[0]);
+          }
+          if (!(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err))) break;
+          fence_after();
+          issue_o(1, Lv, j > 0);
+          mma_commit(&bar_empty[Lv % C::kStages]);
+          if (more) {
+            issue_s(1, Lk);
+            mma_commit(&bar_s[1]);
+            mma_commit(&bar_empty[Lk % C::kStages]);
+          }
+        }
+        // Completes once every MMA issued above has finished (also on abort),
+        // so TMEM is quiet before it is freed.
+        mma_commit(&bar_o);
+        mbar_wait(&bar_o, 0, &abort_flag, a.err, false);
       }
-      // Completes once every MMA issued above has finished (also on abort),
-      // so TMEM is quiet before it is freed.
-      mma_commit(&bar_o);
-      mbar_wait(&bar_o, 0, &abort_flag, a.err, false);
+      __syncwarp();
     }
-    __syncwarp();
+    fence_before();
+    named_barrier_sync(1, kTcThreads);
+    if (warp == 1) {
+      fence_after();
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                   "r"(kTmemCols)
+                   : "memory");
+    }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsHigh));
     // ------------------------------------------------ softmax / epilogue
-    const int t = (warp - 2) >> 2;
+    const int t = (warp - 4) >> 2;
     const int wq = warp & 3;                       // TMEM lane quarter of this warp
     const int r = wq * 32 + lane;                  // row within the Q tile
     const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
@@ -517,15 +583,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         }
       }
     }
-  }
-
-  fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
-                 "r"(kTmemCols)
-                 : "memory");
+    fence_before();
+    named_barrier_sync(1, kTcThreads);
   }
 }
 
@@ -654,6 +713,12 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return HSA_ERR_CUDA;
   if (!configured[dev].load()) {
+    // The register hand-over inside the kernel assumes exactly kLaunchRegs
+    // registers per thread at launch; any other count could leave the
+    // softmax warps waiting for registers, so refuse to launch.
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, attn_tc_kernel<D>) != cudaSuccess) return HSA_ERR_CUDA;
+    if (fa.numRegs != kLaunchRegs || fa.maxThreadsPerBlock < kTcThreads) return HSA_ERR_UNSUPPORTED;
     if (cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::kSmem) != cudaSuccess)
       return HSA_ERR_CUDA;
