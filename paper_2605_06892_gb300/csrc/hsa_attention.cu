@@ -72,6 +72,18 @@ __device__ __forceinline__ bool mbar_test(uint64_t *b, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of phase `parity` (never suspends the thread).
+__device__ __forceinline__ bool mbar_peek(uint64_t *b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(b)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // try_wait that lets the hardware suspend the thread for up to ~0.5 ms while
 // the phase is incomplete, so waiting warps take no issue slots from the
 // working ones.
@@ -471,55 +483,75 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         const uint64_t dk0 = sdesc(kv_base, 16, 1024);
         const uint64_t dv0 = sdesc(kv_base, kBN * 128, 1024);
         constexpr uint32_t kTile16 = C::kTileBytes >> 4;
+        // The tensor pipe queues only a few MMAs, so the issuing thread must
+        // not stop with an empty queue.  Each group of eight MMAs therefore
+        // issues six, then `peek`s (non-blocking) the barriers the next group
+        // needs while the last queued MMAs still run, then issues the last two;
+        // a barrier found complete needs no blocking wait afterwards.
         // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
-        auto issue_s = [&](int t, int L) {
+        auto issue_s = [&](int t, int L, auto peek) {
           const uint64_t dq = dq0 + t * kTile16;
           const uint64_t dk = dk0 + (L % C::kStages) * kTile16;
           const uint32_t ts = tmem + 128 * t;
 #pragma unroll
           for (int k = 0; k < D / 16; ++k) {
+            if (k == D / 16 - 2) peek();
             const uint32_t off = ((k >> 2) * (kBM * 128) + (k & 3) * 32) >> 4;
             mma_ss(ts, dq + off, dk + off, kIdS, k > 0);
           }
         };
         // O_t += P_t V: P in TMEM (bf16 pairs in the S_t columns), V MN-major.
-        auto issue_o = [&](int t, int L, bool acc) {
+        auto issue_o = [&](int t, int L, bool acc, auto peek) {
           const uint64_t dv = dv0 + (L % C::kStages) * kTile16;
           const uint32_t to = tmem + C::kOCol0 + D * t, tp = tmem + 128 * t;
 #pragma unroll
-          for (int k = 0; k < kBN / 16; ++k)
+          for (int k = 0; k < kBN / 16; ++k) {
+            if (k == kBN / 16 - 2) peek();
             mma_ts(to, tp + 8 * k, dv + ((k * 2048) >> 4), kIdO, (acc || k > 0) ? 1u : 0u);
+          }
+        };
+        auto full_ready = [&](int L) {
+          return mbar_peek(&bar_full[L % C::kStages], (L / C::kStages) & 1);
         };
         bool ok = wait_full(0);
+        bool rdy_v = false, rdy_k = false, rdy_p0 = false, rdy_p1 = false;
         if (ok) {
           fence_after();
-          issue_s(0, 0);
+          issue_s(0, 0, [] {});
           mma_commit(&bar_s[0]);
-          issue_s(1, 0);
+          issue_s(1, 0, [&] { rdy_v = nT > 0 && full_ready(1); });
           mma_commit(&bar_s[1]);
           mma_commit(&bar_empty[0]);
         }
         for (int j = 0; ok && j < nT; ++j) {
           const int Lv = 2 * j + 1, Lk = 2 * j + 2;
           const bool more = j + 1 < nT;
-          if (!(ok = wait_full(Lv))) break;
-          if (!(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err))) break;
+          if (!rdy_v && !(ok = wait_full(Lv))) break;
+          if (!rdy_p0 && !(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err))) break;
           fence_after();
-          issue_o(0, Lv, j > 0);
+          issue_o(0, Lv, j > 0, [&] { rdy_k = more && full_ready(Lk); });
           if (more) {
-            if (!(ok = wait_full(Lk))) break;
+            if (!rdy_k && !(ok = wait_full(Lk))) break;
             fence_after();
-            issue_s(0, Lk);
+            issue_s(0, Lk, [&] { rdy_p1 = mbar_peek(&bar_p[1], j & 1); });
             mma_commit(&bar_s[0]);
+          } else {
+            rdy_p1 = false;
           }
-          if (!(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err))) break;
+          if (!rdy_p1 && !(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err))) break;
           fence_after();
-          issue_o(1, Lv, j > 0);
-          mma_commit(&bar_empty[Lv % C::kStages]);
           if (more) {
-            issue_s(1, Lk);
+            issue_o(1, Lv, j > 0, [] {});
+            mma_commit(&bar_empty[Lv % C::kStages]);
+            issue_s(1, Lk, [&] {
+              rdy_v = full_ready(Lv + 2);
+              rdy_p0 = mbar_peek(&bar_p[0], (j + 1) & 1);
+            });
             mma_commit(&bar_s[1]);
             mma_commit(&bar_empty[Lk % C::kStages]);
+          } else {
+            issue_o(1, Lv, j > 0, [] {});
+            mma_commit(&bar_empty[Lv % C::kStages]);
           }
         }
         // Completes once every MMA issued above has finished (also on abort),
