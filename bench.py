@@ -53,6 +53,8 @@ def parse():
     p.add_argument("--workload", default="wan13b", choices=list(synth.WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--memory-sweep", action="store_true",
+                   help="HBM size sweep of gather, KV scatter and cached Euler (L2 flushed)")
     return p.parse_args()
 
 
@@ -480,8 +482,77 @@ def run_reference(args, dist, rank, world):
     }), flush=True)
 
 
+def memory_sweep():
+    """Gather / KV-scatter / cached-Euler bandwidth from L2-sized to multi-GB
+    footprints.  Each rep is timed alone with CUDA events after an L2 flush;
+    bytes are the algorithmic bytes of the call (see `algorithmic`)."""
+    import paper_2605_06892_gb300 as hsa
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    peaks, src = load_peaks()
+    g = torch.Generator(device="cpu").manual_seed(7)
+
+    def timed(fn, reps=10):
+        for _ in range(3):
+            fn()
+        ts = []
+        for _ in range(reps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts)
+
+    def report(kind, shape, nbytes, ms):
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        print(json.dumps({"sweep": kind, "shape": shape, "bytes": nbytes, "ms": ms, "gbs": gbs,
+                          "frac_hbm": gbs / peaks["hbm_gbs"], "peak_source": src}), flush=True)
+
+    row = 3072                                   # one Wan-1.3B token row, 12 x 128 bf16
+    for n in (8192, 32768, 131072, 262144, 524288):
+        N = 2 * n
+        src_t = torch.empty((N, row // 2), dtype=torch.bfloat16, device=dev).normal_()
+        idx = torch.randperm(N, generator=g)[:n].sort().values.to(torch.int32).to(dev)
+        dst = torch.empty((n, row // 2), dtype=torch.bfloat16, device=dev)
+        ms = timed(lambda: hsa.hsa_gather_active(src_t, idx, n, dst, stream))
+        report("gather", f"{n} rows x {row} B", n * (2 * row + 4), ms)
+        del src_t, dst
+        kc = torch.empty((N, 12, 128), dtype=torch.bfloat16, device=dev).normal_()
+        vc = torch.empty_like(kc).normal_()
+        kf = torch.empty((n, 12, 128), dtype=torch.bfloat16, device=dev).normal_()
+        vf = torch.empty_like(kf).normal_()
+        ms = timed(lambda: hsa.hsa_kv_sync_scatter(kc, vc, kf, vf, idx, n, stream))
+        report("kv_scatter", f"{n} rows x 2 x {row} B", n * (4 * row + 4), ms)
+        del kc, vc, kf, vf
+    for C in (16, 128):
+        for N in (1 << 16, 1 << 20, 1 << 22, 1 << 24):
+            if N * C * 4 > (1 << 31):
+                continue
+            n = N // 2
+            x = torch.empty((N, C), device=dev).normal_()
+            vh = torch.empty_like(x).normal_()
+            vfr = torch.empty((n, C), device=dev).normal_()
+            pos = torch.full((N,), -1, dtype=torch.int32)
+            act = torch.randperm(N, generator=g)[:n].sort().values
+            pos[act] = torch.arange(n, dtype=torch.int32)
+            pos = pos.to(dev)
+            ms = timed(lambda: hsa.hsa_cached_euler(x, vh, vfr, pos, -0.025, n, stream))
+            nbytes = (N - n) * 12 * C + n * 16 * C + 4 * N
+            report("cached_euler", f"N={N} C={C}, half active", nbytes, ms)
+            del x, vh, vfr, pos
+    assert hsa.hsa_get_device_error(stream) == 0
+
+
 def main():
     args = parse()
+    if args.memory_sweep:
+        memory_sweep()
+        return
     if args.impl == "reference":
         dist, rank, world, _ = dist_setup("gloo")
         run_reference(args, dist, rank, world)

@@ -5,7 +5,7 @@
 // All three move whole token rows.  A row is split into 16-byte vectors and a
 // group of L lanes (L a power of two <= 32) of one warp cooperates on a row, so
 // a warp covers 32/L rows at once and every access is a coalesced 128-bit load
-// or store.  Each lane keeps up to kUnroll vectors in flight before storing.
+// or store.  Each lane keeps several vectors in flight before storing.
 // The row index is read once per row by its lane group; indices are checked
 // against the row count and a bad one skips its row and sets the error word.
 #include "hsa_internal.cuh"
@@ -14,7 +14,12 @@ namespace hsa {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kUnroll = 4;
+// 16-byte vectors each lane keeps in flight (measured on GB300 with an L2-
+// flushed size sweep: the gather reaches its best rate at 4, the scatter,
+// whose loads are contiguous, at 8; Euler holds two vectors per step).
+constexpr int kGatherUnroll = 4;
+constexpr int kScatterUnroll = 8;
+constexpr int kEulerUnroll = 4;  // float4 positions per thread per pass (large N)
 
 __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
   uint4 v;
@@ -26,7 +31,7 @@ __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
 // Row loop shared by gather and scatter: rows are handed out to lane groups
 // in a grid-stride loop; `map(j, s, d)` sets the source and destination row
 // pointers of row j, or returns false to skip the row.
-template <class RowMap>
+template <int kUnroll, class RowMap>
 __device__ __forceinline__ void copy_rows(long long n_rows, int vecs, int lpr_log2,
                                           RowMap map) {
   const int L = 1 << lpr_log2;
@@ -60,7 +65,7 @@ __global__ void __launch_bounds__(kThreads)
 gather_rows_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
               const int32_t *__restrict__ idx, int n_active, int N, int vecs,
               int lpr_log2, unsigned *err) {
-  copy_rows(n_active, vecs, lpr_log2, [&](long long j, const uint4 *&s, uint4 *&d) {
+  copy_rows<kGatherUnroll>(n_active, vecs, lpr_log2, [&](long long j, const uint4 *&s, uint4 *&d) {
     const int r = __ldg(idx + j);
     if (r < 0 || r >= N) {
       set_error(err, kErrIndex);
@@ -79,7 +84,7 @@ kv_scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
                const uint4 *__restrict__ kf, const uint4 *__restrict__ vf,
                const int32_t *__restrict__ idx, int n_active, int N, int vecs,
                int lpr_log2, unsigned *err) {
-  copy_rows(2LL * n_active, vecs, lpr_log2, [&](long long jj, const uint4 *&s, uint4 *&d) {
+  copy_rows<kScatterUnroll>(2LL * n_active, vecs, lpr_log2, [&](long long jj, const uint4 *&s, uint4 *&d) {
     const bool is_v = jj >= n_active;
     const long long j = is_v ? jj - n_active : jj;
     const int r = __ldg(idx + j);
@@ -94,56 +99,63 @@ kv_scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
 }
 
 // x[n] = fma(vhat[n], dsigma, x[n]) with vhat[n] refreshed from
-// v_fresh[pos[n]] when pos[n] >= 0.  A row is C/4 float4 vectors.
+// v_fresh[pos[n]] when pos[n] >= 0.  Element-wise over the N*C/4 float4
+// vectors: each thread takes kEulerUnroll vectors a grid-stride apart, loads
+// their pos entries, then all their x and velocity vectors, then stores, so
+// 3*kEulerUnroll independent loads are in flight per thread whatever C is.
+// vec_shift = log2(C/4) when C/4 is a power of two, else -1 (division).
+// Small N uses one vector per thread (kU = 1) so that every SM has work.
+template <int kU>
 __global__ void __launch_bounds__(kThreads)
 cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
-             const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
-             int N, int vecs, int lpr_log2, float dsigma, int n_fresh_rows, unsigned *err) {
-  const int L = 1 << lpr_log2;
-  const int lane = threadIdx.x & 31;
-  const int sub = lane >> lpr_log2;
-  const int sl = lane & (L - 1);
-  const int rows_per_warp = 32 >> lpr_log2;
-  const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
-  const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-  for (long long n = warp * rows_per_warp + sub; n < N; n += nwarps * rows_per_warp) {
-    int p = pos ? __ldg(pos + n) : -1;
-    if (p >= n_fresh_rows) {
-      set_error(err, kErrIndex);
-      p = -1;
-    }
-    float4 *xr = x + n * vecs;
-    float4 *vr = vhat + n * vecs;
-    const float4 *src = p >= 0 ? v_fresh + (long long)p * vecs : vr;
-    for (int v0 = sl; v0 < vecs; v0 += kUnroll * L) {
-      float4 vb[kUnroll], xb[kUnroll];
+                    const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
+                    long long total, int vecs, int vec_shift, float dsigma, int n_fresh_rows,
+                    unsigned *err) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long base = blockIdx.x * (long long)blockDim.x + threadIdx.x; base < total;
+       base += stride * kU) {
+    long long e[kU], row[kU];
+    int p[kU];
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int v = v0 + u * L;
-        if (v < vecs) {
-          vb[u] = src[v];
-          xb[u] = xr[v];
+    for (int u = 0; u < kU; ++u) {
+      e[u] = base + u * stride;
+      row[u] = vec_shift >= 0 ? (e[u] >> vec_shift) : e[u] / vecs;
+      p[u] = -1;
+      if (pos && e[u] < total) {
+        p[u] = __ldg(pos + row[u]);
+        if (p[u] >= n_fresh_rows) {
+          set_error(err, kErrIndex);
+          p[u] = -1;
         }
       }
+    }
+    float4 vb[kU], xb[kU];
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int v = v0 + u * L;
-        if (v < vecs) {
-          if (p >= 0) vr[v] = vb[u];
-          float4 o;
-          o.x = __fmaf_rn(vb[u].x, dsigma, xb[u].x);
-          o.y = __fmaf_rn(vb[u].y, dsigma, xb[u].y);
-          o.z = __fmaf_rn(vb[u].z, dsigma, xb[u].z);
-          o.w = __fmaf_rn(vb[u].w, dsigma, xb[u].w);
-          xr[v] = o;
-        }
+    for (int u = 0; u < kU; ++u) {
+      if (e[u] < total) {
+        const long long c = e[u] - row[u] * vecs;
+        vb[u] = p[u] >= 0 ? __ldg(v_fresh + (long long)p[u] * vecs + c) : vhat[e[u]];
+        xb[u] = x[e[u]];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      if (e[u] < total) {
+        if (p[u] >= 0) vhat[e[u]] = vb[u];
+        float4 o;
+        o.x = __fmaf_rn(vb[u].x, dsigma, xb[u].x);
+        o.y = __fmaf_rn(vb[u].y, dsigma, xb[u].y);
+        o.z = __fmaf_rn(vb[u].z, dsigma, xb[u].z);
+        o.w = __fmaf_rn(vb[u].w, dsigma, xb[u].w);
+        x[e[u]] = o;
       }
     }
   }
 }
 
-// Grid for n_rows rows handled by lane groups of size L: enough warps to give
-// every SM a full complement of resident threads, no more than the rows need.
+// Grid for n_rows rows handled by lane groups of size L: up to 8 blocks of
+// 256 threads per SM (a full SM), no more than the rows need; blocks beyond
+// what is resident wait their turn.
 int grid_for(long long n_rows, int L) {
   const long long rows_per_block = (long long)(kThreads / 32) * (32 / L);
   long long blocks = (n_rows + rows_per_block - 1) / rows_per_block;
@@ -213,9 +225,22 @@ extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   const int vecs = C / 4;
-  const int L = lanes_per_row(vecs);
-  cached_euler_kernel<<<grid_for(N, L), kThreads, 0, (cudaStream_t)stream>>>(
-      (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, N, vecs, log2i(L), dsigma,
-      pos ? n_fresh : 0, err);
+  const long long total = (long long)N * vecs;
+  int vec_shift = -1;
+  for (int sh = 0; sh < 31; ++sh)
+    if ((1 << sh) == vecs) vec_shift = sh;
+  const long long resident = (long long)sm_count() * 2048;     // threads
+  const int per = total >= (long long)kEulerUnroll * resident ? kEulerUnroll : 1;
+  long long blocks = (total + (long long)kThreads * per - 1) / ((long long)kThreads * per);
+  const long long cap = (long long)sm_count() * (2048 / kThreads);
+  if (blocks > cap) blocks = cap;
+  if (per == kEulerUnroll)
+    cached_euler_kernel<kEulerUnroll><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
+        (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
+        dsigma, pos ? n_fresh : 0, err);
+  else
+    cached_euler_kernel<1><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
+        (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
+        dsigma, pos ? n_fresh : 0, err);
   return launch_status();
 }

@@ -420,6 +420,20 @@ def test_cached_euler_workloads(hsa, name):
     _no_device_error(hsa)
 
 
+@pytest.mark.parametrize("N,C", [(777, 12), (1000, 20), (5, 4), (33333, 8)])
+def test_cached_euler_odd_widths(hsa, N, C):
+    """C/4 not a power of two (division path), tiny N, ragged N."""
+    g = torch.Generator().manual_seed(N)
+    x = synth.normal((N, C), 1)
+    vh = synth.normal((N, C), 2)
+    idx = synth.uniform_subset(N, max(1, N // 3), 3)
+    pos = torch.full((N,), -1, dtype=torch.int32)
+    pos[idx.long()] = torch.arange(idx.numel(), dtype=torch.int32)
+    vfr = synth.normal((idx.numel(), C), 4)
+    _euler_step_check(hsa, x, vh, vfr, pos, -0.0625)
+    _no_device_error(hsa)
+
+
 def test_cached_euler_skip4_telescopes(hsa):
     """Tiny workload, skip length 4: four cached steps of the GPU equal the
     fp32 mirror bit for bit and one fp64 Euler step from sigma_i to
