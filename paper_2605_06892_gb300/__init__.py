@@ -22,7 +22,7 @@ __all__ = [
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
     "hsa_partition", "hsa_partition_static", "hsa_partition_active", "hsa_gather_active",
     "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_cached_euler",
-    "hsa_get_device_error",
+    "hsa_get_device_error", "hsa_test_inject_attention_stall",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -64,6 +64,7 @@ _SIGS = {
                               _c_p, _c_int, _c_p], _c_int),
     "hsa_cached_euler": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p], _c_int),
     "hsa_get_device_error": ([_c_p], _c_int),
+    "hsa_test_inject_attention_stall": ([_c_int], _c_int),
 }
 
 _lib = None
@@ -224,3 +225,10 @@ def hsa_cached_euler(x, v_cache, v_fresh, pos, dsigma: float, n_fresh: int | Non
 def hsa_get_device_error(stream=None) -> int:
     """Status of the device-side checks since the last call (synchronises)."""
     return lib().hsa_get_device_error(_stream(stream))
+
+
+def hsa_test_inject_attention_stall(mode: int) -> int:
+    """Test hook (include/hsa_test.h): mode 1 makes following bf16 attention
+    launches withhold one internal signal so their bounded wait runs out and
+    HSA_ERR_TIMEOUT is reported; mode 0 restores normal operation."""
+    return _check(lib().hsa_test_inject_attention_stall(mode), "hsa_test_inject_attention_stall")

@@ -36,6 +36,7 @@
 #include <cmath>
 
 #include "hsa_internal.cuh"
+#include "hsa_test.h"
 
 namespace hsa {
 namespace {
@@ -295,6 +296,7 @@ struct TcArgs {
   unsigned *err;
   int n_active, N, H, q_rows, n_kv_tiles;
   float scale_log2;
+  int inject_stall;   // test hook (hsa_test.h): 1 = tile 0 withholds its first P
 };
 
 // Scores of one 128-key tile for this thread's row: S from TMEM (one read),
@@ -591,7 +593,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         softmax_tile<D, true>(tS, tO, valid, j == 0, sl2, m_run, l_run);
       tmem_wait_st();
       fence_before();
-      mbar_arrive(&bar_p[t]);
+      if (!(a.inject_stall == 1 && t == 0 && j == 0)) mbar_arrive(&bar_p[t]);
     }
     if (ok && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
       fence_after();
@@ -705,6 +707,8 @@ attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
 
 // -------------------------------------------------------------- host side
 
+std::atomic<int> g_inject_stall{0};
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static std::atomic<PFN_cuTensorMapEncodeTiled_v12000> fn{nullptr};
   PFN_cuTensorMapEncodeTiled_v12000 f = fn.load();
@@ -770,6 +774,7 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.q_rows = q_idx ? N : n_active;
   a.n_kv_tiles = (N + kBN - 1) / kBN;
   a.scale_log2 = scale * 1.4426950408889634f;
+  a.inject_stall = g_inject_stall.load(std::memory_order_relaxed);
   const dim3 grid((n_active + kBM * kQT - 1) / (kBM * kQT), H);
   attn_tc_kernel<D><<<grid, kTcThreads, C::kSmem, stream>>>(mk, mv, a);
   return launch_status();
@@ -817,4 +822,9 @@ extern "C" int hsa_active_attention(const void *q, const int32_t *q_idx, int n_a
                     : launch_tc<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
   return D == 128 ? launch_f32<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err)
                   : launch_f32<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
+}
+
+extern "C" int hsa_test_inject_attention_stall(int mode) {
+  if (mode != 0 && mode != 1) return HSA_ERR_INVALID_ARG;
+  return g_inject_stall.exchange(mode);
 }
