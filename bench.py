@@ -214,6 +214,9 @@ def run_hsa(args, dist, rank, world, local_rank):
     T, budgets = w.T, w.budgets
     sig = hsa.hsa_sigma_schedule(T, w.shift)
     ws = torch.empty(hsa.hsa_partition_workspace_bytes(w.N), dtype=torch.uint8, device=dev)
+    ws_att = torch.empty(max(1, hsa.hsa_active_attention_workspace_bytes(
+        w.N, w.N, w.H, w.D, 0 if w.dtype == "bf16" else 1)), dtype=torch.uint8, device=dev)
+    L.ws_att = ws_att
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     n_of = {it: hsa.hsa_active_count(budgets, L.counts, T, it, w.window_pct) for it in L.iters}
@@ -235,7 +238,7 @@ def run_hsa(args, dist, rank, world, local_rank):
             record("scatter", lambda: hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, n,
                                                               stream))
             record("attention", lambda: hsa.hsa_active_attention(L.q, L.idx, n, L.kc, L.vc,
-                                                                 L.out, 0.0, stream))
+                                                                 L.out, 0.0, ws_att, stream))
             record("euler", lambda: hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n,
                                                          stream))
 
@@ -358,7 +361,7 @@ def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
                                      stream)
             hsa.hsa_gather_active(L.hidden, L.idx, n, L.gathered, stream)
             hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, n, stream)
-            hsa.hsa_active_attention(d_q, None, n, L.kc, L.vc, L.out, 0.0, stream)
+            hsa.hsa_active_attention(d_q, None, n, L.kc, L.vc, L.out, 0.0, L.ws_att, stream)
             h_out[:n].copy_(L.out[:n], non_blocking=True)
             hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n, stream)
         h_x.copy_(L.x, non_blocking=True)

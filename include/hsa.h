@@ -198,14 +198,29 @@ int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_fresh,
  * O(|A_i| N) instead of O(N^2).
  *   k_cache, v_cache  device, [N, H, D] of dtype.
  *   out               device, [n_active, H, D] of dtype, written.
+ *   workspace         device, optional (NULL = none), 16-byte aligned; see
+ *                     hsa_active_attention_workspace_bytes.  With it, the
+ *                     (query block, head) units of the last, partly filled
+ *                     wave of CTAs are split along the keys and merged
+ *                     afterwards, so that wave runs as full as the others;
+ *                     without it the result is the same up to rounding order.
+ *                     Overwritten; calls using one workspace must not overlap.
  * Supported: D in {64, 128}; H >= 1; 1 <= N < 2^31; 0 <= n_active.
  * HSA_BF16 runs on the tensor cores (tcgen05, fp32 accumulation); HSA_F32
- * runs in fp32 on the CUDA cores.  Pointers must be 16-byte aligned.  A q_idx
- * entry outside [0, N) yields a zero query row (HSA_ERR_INDEX). */
+ * runs in fp32 on the CUDA cores and ignores the workspace.  Pointers must be
+ * 16-byte aligned.  A q_idx entry outside [0, N) yields a zero query row
+ * (HSA_ERR_INDEX). */
 int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
                          const void *k_cache, const void *v_cache, int N, int H,
                          int D, float scale, void *out, hsa_dtype dtype,
+                         void *workspace, size_t workspace_bytes,
                          hsa_stream_t stream);
+
+/* Workspace bytes that let hsa_active_attention balance its last wave (0 when
+ * the dtype or shape takes none).  Depends only on the device's SM count and
+ * D, so one buffer serves every call of a given D on that device. */
+size_t hsa_active_attention_workspace_bytes(int n_active, int N, int H, int D,
+                                            hsa_dtype dtype);
 
 /* ------------------------------------------------------- a6 cached Euler */
 

@@ -21,7 +21,8 @@ __all__ = [
     "hsa_status_string", "hsa_version", "hsa_check_budgets", "hsa_window_margin",
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
     "hsa_partition", "hsa_partition_static", "hsa_partition_active", "hsa_gather_active",
-    "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_cached_euler",
+    "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_active_attention_workspace_bytes",
+    "hsa_cached_euler",
     "hsa_get_device_error", "hsa_test_inject_attention_stall",
 ]
 
@@ -61,7 +62,8 @@ _SIGS = {
     "hsa_kv_sync_scatter": ([_c_p, _c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_int,
                              _c_int, _c_p], _c_int),
     "hsa_active_attention": ([_c_p, _c_p, _c_int, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f,
-                              _c_p, _c_int, _c_p], _c_int),
+                              _c_p, _c_int, _c_p, _c_sz, _c_p], _c_int),
+    "hsa_active_attention_workspace_bytes": ([_c_int, _c_int, _c_int, _c_int, _c_int], _c_sz),
     "hsa_cached_euler": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p], _c_int),
     "hsa_get_device_error": ([_c_p], _c_int),
     "hsa_test_inject_attention_stall": ([_c_int], _c_int),
@@ -203,14 +205,22 @@ def hsa_kv_sync_scatter(k_cache, v_cache, k_fresh, v_fresh, idx, n_active: int,
                                      _stream(stream)), "hsa_kv_sync_scatter")
 
 
+def hsa_active_attention_workspace_bytes(n_active: int, N: int, H: int, D: int,
+                                         dtype: int = HSA_BF16) -> int:
+    return lib().hsa_active_attention_workspace_bytes(n_active, N, H, D, dtype)
+
+
 def hsa_active_attention(q, q_idx, n_active: int, k_cache, v_cache, out, scale: float = 0.0,
-                         stream=None) -> None:
+                         workspace=None, stream=None) -> None:
     """out[j] = attention of query row q_idx[j] (q: [N,H,D]) or j (q_idx None,
-    q: [n_active,H,D]) against the full cache."""
+    q: [n_active,H,D]) against the full cache; `workspace` (optional uint8
+    device tensor) lets the last wave of CTAs be split along the keys."""
     N, H, D = k_cache.shape
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     _check(lib().hsa_active_attention(_p(q), _p(q_idx), n_active, _p(k_cache), _p(v_cache), N,
                                       H, D, float(scale), _p(out), _dtype_code(k_cache),
-                                      _stream(stream)), "hsa_active_attention")
+                                      _p(workspace), ws_bytes, _stream(stream)),
+           "hsa_active_attention")
 
 
 def hsa_cached_euler(x, v_cache, v_fresh, pos, dsigma: float, n_fresh: int | None = None,

@@ -297,7 +297,41 @@ struct TcArgs {
   int n_active, N, H, q_rows, n_kv_tiles;
   float scale_log2;
   int inject_stall;   // test hook (hsa_test.h): 1 = tile 0 withholds its first P
+  // Work split.  CTA b < n_whole owns unit b (head b / n_qblocks, query block
+  // b % n_qblocks) over all key tiles.  Every later CTA owns one of `pieces`
+  // key ranges of a tail unit and writes its unnormalised O, running maximum
+  // and sum to ws_o / ws_ml for the combine kernel.
+  int n_qblocks, n_whole, pieces;
+  float *ws_o;        // [piece CTA][kQT*kBM rows][D] fp32
+  float *ws_ml;       // [piece CTA][kQT*kBM rows][2] fp32: m (log2 units), l
 };
+
+// Key-tile range [j0, j1) and unit of CTA b.
+struct CtaWork {
+  int head, row0, j0, j1, piece;   // piece = -1 for a whole unit
+};
+
+__host__ __device__ inline CtaWork cta_work(int b, int n_qblocks, int n_whole, int pieces,
+                                            int n_kv_tiles) {
+  CtaWork w;
+  int unit;
+  if (b < n_whole) {
+    unit = b;
+    w.j0 = 0;
+    w.j1 = n_kv_tiles;
+    w.piece = -1;
+  } else {
+    const int pi = b - n_whole;
+    unit = n_whole + pi / pieces;
+    const int k = pi % pieces;
+    w.j0 = (int)((long long)n_kv_tiles * k / pieces);
+    w.j1 = (int)((long long)n_kv_tiles * (k + 1) / pieces);
+    w.piece = pi;
+  }
+  w.head = unit / n_qblocks;
+  w.row0 = (unit % n_qblocks) * (kBM * kQT);
+  return w;
+}
 
 // Scores of one 128-key tile for this thread's row: S from TMEM (one read),
 // the running maximum (moved only when it grows by more than 2^8, with O
@@ -391,9 +425,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.y;
-  const int row0 = blockIdx.x * (kBM * kQT);
-  const int nT = a.n_kv_tiles;
+  const CtaWork wk = cta_work(blockIdx.x, a.n_qblocks, a.n_whole, a.pieces, a.n_kv_tiles);
+  const int h = wk.head;
+  const int row0 = wk.row0;
+  const int j0 = wk.j0;
+  const int nT = wk.j1 - wk.j0;        // key tiles of this CTA (local index j = 0..nT-1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -461,7 +497,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
           uint8_t *dst = sKV + slot * C::kTileBytes;
 #pragma unroll
           for (int c = 0; c < C::kChunks; ++c)
-            tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, (L >> 1) * kBN);
+            tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64,
+                        (j0 + (L >> 1)) * kBN);
           issued = L + 1;
         }
         // Drain: every issued copy has landed before the CTA may exit.
@@ -586,7 +623,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     for (int j = 0; j < nT; ++j) {
       if (!(ok = mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err))) break;
       fence_after();
-      const int valid = a.N - j * kBN;             // keys of this tile that exist
+      const int valid = a.N - (j0 + j) * kBN;      // keys of this tile that exist
       if (valid >= kBN)
         softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
       else
@@ -595,7 +632,25 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       fence_before();
       if (!(a.inject_stall == 1 && t == 0 && j == 0)) mbar_arrive(&bar_p[t]);
     }
-    if (ok && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
+    if (ok && wk.piece >= 0 && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
+      // Piece of a split unit: unnormalised O, maximum and sum, for the combine.
+      fence_after();
+      const int prow = t * kBM + r;
+      float *po = a.ws_o + ((size_t)wk.piece * (kQT * kBM) + prow) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tO + 32 * c, o);
+        tmem_wait_ld();
+        float4 *d4 = reinterpret_cast<float4 *>(po + 32 * c);
+#pragma unroll
+        for (int v = 0; v < 8; ++v)
+          d4[v] = make_float4(__uint_as_float(o[4 * v]), __uint_as_float(o[4 * v + 1]),
+                              __uint_as_float(o[4 * v + 2]), __uint_as_float(o[4 * v + 3]));
+      }
+      reinterpret_cast<float2 *>(a.ws_ml)[(size_t)wk.piece * (kQT * kBM) + prow] =
+          make_float2(m_run, l_run);
+    } else if (ok && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
       fence_after();
       const int grow = row0 + t * kBM + r;
       const float inv = 1.f / l_run;
@@ -620,6 +675,44 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     fence_before();
     named_barrier_sync(1, kTcThreads);
   }
+}
+
+// ------------------------------------------------------ split-unit combine
+//
+// One warp per (tail unit, row): merge the unit's key-range pieces,
+// O = sum_p 2^(m_p - M) O_p / sum_p 2^(m_p - M) l_p with M = max_p m_p, and
+// store the bf16 row.  Lanes stride over D, so every access is coalesced.
+template <int D>
+__global__ void __launch_bounds__(256)
+attn_combine_kernel(const float *__restrict__ ws_o, const float *__restrict__ ws_ml, int n_tail,
+                    int n_whole, int pieces, int n_qblocks, int n_active, int H,
+                    __nv_bfloat16 *__restrict__ out) {
+  constexpr int kRows = kQT * kBM;
+  const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  const int u = wid / kRows, row = wid % kRows;
+  if (u >= n_tail) return;
+  const int unit = n_whole + u;
+  const int head = unit / n_qblocks;
+  const int grow = (unit % n_qblocks) * kRows + row;
+  if (grow >= n_active) return;
+  const float2 *ml = reinterpret_cast<const float2 *>(ws_ml);
+  float M = -INFINITY;
+  for (int p = 0; p < pieces; ++p) M = fmaxf(M, ml[((size_t)u * pieces + p) * kRows + row].x);
+  float L = 0.f, acc[D / 32];
+#pragma unroll
+  for (int i = 0; i < D / 32; ++i) acc[i] = 0.f;
+  for (int p = 0; p < pieces; ++p) {
+    const size_t pr = ((size_t)u * pieces + p) * kRows + row;
+    const float2 v = ml[pr];
+    const float w = exp2f(v.x - M);
+    L = fmaf(w, v.y, L);
+#pragma unroll
+    for (int i = 0; i < D / 32; ++i) acc[i] = fmaf(w, ws_o[pr * D + lane + 32 * i], acc[i]);
+  }
+  const float inv = 1.f / L;
+  __nv_bfloat16 *dst = out + ((size_t)grow * H + head) * D;
+#pragma unroll
+  for (int i = 0; i < D / 32; ++i) dst[lane + 32 * i] = __float2bfloat16_rn(acc[i] * inv);
 }
 
 // ------------------------------------------------------ fp32 CUDA-core kernel
@@ -740,10 +833,16 @@ bool make_kv_map(CUtensorMap *map, const void *base, int N, int H, int D) {
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Bytes of split-unit workspace for head dimension D: at most one piece per
+// SM, kQT*kBM rows each, D fp32 of O plus (m, l).
+size_t split_workspace_bytes(int D) {
+  return (size_t)sm_count() * (kQT * kBM) * ((size_t)D * 4 + 8) + 512;
+}
+
 template <int D>
 int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
-              const void *v_cache, int N, int H, float scale, void *out, cudaStream_t stream,
-              unsigned *err) {
+              const void *v_cache, int N, int H, float scale, void *out, void *ws,
+              size_t ws_bytes, cudaStream_t stream, unsigned *err) {
   using C = TcCfg<D>;
   static std::atomic<int> configured[64];
   int dev = 0;
@@ -775,8 +874,33 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.n_kv_tiles = (N + kBN - 1) / kBN;
   a.scale_log2 = scale * 1.4426950408889634f;
   a.inject_stall = g_inject_stall.load(std::memory_order_relaxed);
-  const dim3 grid((n_active + kBM * kQT - 1) / (kBM * kQT), H);
-  attn_tc_kernel<D><<<grid, kTcThreads, C::kSmem, stream>>>(mk, mv, a);
+  // Work plan: one CTA per SM at a time, so U units take ceil(U / sms) waves.
+  // With a workspace, the rem = U mod sms units of the last wave are split
+  // along the keys into `pieces` ranges that fill that wave, then combined.
+  a.n_qblocks = (n_active + kQT * kBM - 1) / (kQT * kBM);
+  const long long units = (long long)a.n_qblocks * H;
+  if (units > 0x7fffffffLL) return HSA_ERR_UNSUPPORTED;
+  const int sms = sm_count();
+  const int rem = (int)(units % sms);
+  int pieces = 1;
+  if (ws && rem > 0) {
+    pieces = sms / rem;
+    if (pieces > a.n_kv_tiles) pieces = a.n_kv_tiles;
+    const size_t need = (size_t)rem * pieces * (kQT * kBM) * ((size_t)D * 4 + 8);
+    if (pieces < 2 || need > ws_bytes || (reinterpret_cast<uintptr_t>(ws) & 15)) pieces = 1;
+  }
+  a.pieces = pieces;
+  a.n_whole = pieces > 1 ? (int)(units - rem) : (int)units;
+  a.ws_o = pieces > 1 ? static_cast<float *>(ws) : nullptr;
+  a.ws_ml = pieces > 1 ? a.ws_o + (size_t)rem * pieces * (kQT * kBM) * D : nullptr;
+  const long long grid = (long long)a.n_whole + (pieces > 1 ? (long long)rem * pieces : 0);
+  attn_tc_kernel<D><<<(unsigned)grid, kTcThreads, C::kSmem, stream>>>(mk, mv, a);
+  if (cudaGetLastError() != cudaSuccess) return HSA_ERR_CUDA;
+  if (pieces > 1) {
+    const long long warps = (long long)rem * (kQT * kBM);
+    attn_combine_kernel<D><<<(unsigned)((warps * 32 + 255) / 256), 256, 0, stream>>>(
+        a.ws_o, a.ws_ml, rem, a.n_whole, pieces, a.n_qblocks, n_active, H, a.out);
+  }
   return launch_status();
 }
 
@@ -798,9 +922,16 @@ int launch_f32(const void *q, const int32_t *q_idx, int n_active, const void *k_
 
 using namespace hsa;
 
+extern "C" size_t hsa_active_attention_workspace_bytes(int n_active, int N, int H, int D,
+                                                      hsa_dtype dtype) {
+  if (dtype != HSA_BF16 || (D != 64 && D != 128) || n_active <= 0 || N <= 0 || H <= 0) return 0;
+  return split_workspace_bytes(D);
+}
+
 extern "C" int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
                                     const void *k_cache, const void *v_cache, int N, int H,
                                     int D, float scale, void *out, hsa_dtype dtype,
+                                    void *workspace, size_t workspace_bytes,
                                     hsa_stream_t stream) {
   if (n_active < 0 || N < 1 || H < 1) return HSA_ERR_INVALID_ARG;
   if (dtype != HSA_BF16 && dtype != HSA_F32) return HSA_ERR_INVALID_ARG;
@@ -818,8 +949,10 @@ extern "C" int hsa_active_attention(const void *q, const int32_t *q_idx, int n_a
   if ((long long)(n_active + kBM * kQT - 1) / (kBM * kQT) > 0x7fffffffLL) return HSA_ERR_UNSUPPORTED;
   if (H > 65535) return HSA_ERR_UNSUPPORTED;
   if (dtype == HSA_BF16)
-    return D == 128 ? launch_tc<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err)
-                    : launch_tc<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
+    return D == 128 ? launch_tc<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out,
+                                     workspace, workspace_bytes, s, err)
+                    : launch_tc<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out,
+                                    workspace, workspace_bytes, s, err);
   return D == 128 ? launch_f32<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err)
                   : launch_f32<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
 }

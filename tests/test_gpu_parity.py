@@ -249,17 +249,28 @@ def test_scatter_canaries_and_bad_index(hsa):
 
 # --------------------------------------------------------------- attention
 
+def _workspace(hsa, n_act, N, H, D, dtype):
+    nbytes = hsa.hsa_active_attention_workspace_bytes(n_act, N, H, D,
+                                                      0 if dtype == "bf16" else 1)
+    return torch.empty(max(nbytes, 1), dtype=torch.uint8, device=DEV)
+
+
 def _attention_case(hsa, N, H, D, n_act, dtype, indexed, seed):
+    """Both launch plans: without a workspace (every unit whole) and with one
+    (last wave split along the keys and combined)."""
     q = synth.normal((N if indexed else n_act, H, D), seed, dtype)
     kc = synth.normal((N, H, D), seed + 1, dtype)
     vc = synth.normal((N, H, D), seed + 2, dtype)
     idx = synth.uniform_subset(N, n_act, seed + 3) if indexed else None
-    out = torch.full((n_act, H, D), 777.0, device=DEV).to(q.dtype)
-    hsa.hsa_active_attention(q.to(DEV), None if idx is None else idx.to(DEV), n_act,
-                             kc.to(DEV), vc.to(DEV), out)
     ref = oracle.attention(q, kc, vc, q_idx=idx)
-    _no_device_error(hsa)
-    return _check_attention(out, ref, dtype)
+    res = None
+    for ws in (None, _workspace(hsa, n_act, N, H, D, dtype)):
+        out = torch.full((n_act, H, D), 777.0, device=DEV).to(q.dtype)
+        hsa.hsa_active_attention(q.to(DEV), None if idx is None else idx.to(DEV), n_act,
+                                 kc.to(DEV), vc.to(DEV), out, workspace=ws)
+        _no_device_error(hsa)
+        res = _check_attention(out, ref, dtype)
+    return res
 
 
 @pytest.mark.parametrize("N,H,D,n_act,dtype,indexed", [
@@ -303,10 +314,13 @@ def test_attention_large_scores_rescale(hsa):
 
 
 def _sampled_rows(n_act, k, seed):
+    """k random rows plus rows of the last Q block: its first 4 and last 12
+    (its tail is ragged whenever n_act is not a multiple of 256)."""
     g = torch.Generator().manual_seed(seed)
     rows = set(torch.randperm(n_act, generator=g)[:k].tolist())
-    last = (n_act - 1) // 256 * 256           # every row of the last Q block
-    rows.update(range(last, n_act))
+    last = (n_act - 1) // 256 * 256
+    rows.update(range(last, min(last + 4, n_act)))
+    rows.update(range(max(last, n_act - 12), n_act))
     return sorted(rows)
 
 
@@ -321,18 +335,31 @@ def _attention_full_size(hsa, name, it, n_rows=24, n_heads=2, seed=0):
     q = synth.normal((w.N, w.H, w.D), 201, w.dtype)
     kc = synth.normal((w.N, w.H, w.D), 202, w.dtype)
     vc = synth.normal((w.N, w.H, w.D), 203, w.dtype)
-    out = torch.empty((n, w.H, w.D), dtype=q.dtype, device=DEV)
-    hsa.hsa_active_attention(q.to(DEV), idx.to(DEV), n, kc.to(DEV), vc.to(DEV), out)
-    _no_device_error(hsa)
-    out = out.cpu()
+    q_d, kc_d, vc_d, idx_d = q.to(DEV), kc.to(DEV), vc.to(DEV), idx.to(DEV)
+    outs = []
+    # the benchmark's launch (with the split-tail workspace) and the plain one
+    for ws in (_workspace(hsa, n, w.N, w.H, w.D, w.dtype), None):
+        out = torch.empty((n, w.H, w.D), dtype=q.dtype, device=DEV)
+        hsa.hsa_active_attention(q_d, idx_d, n, kc_d, vc_d, out, workspace=ws)
+        _no_device_error(hsa)
+        outs.append(out.cpu())
+    del q_d, kc_d, vc_d
     rows = torch.tensor(_sampled_rows(n, n_rows, seed), dtype=torch.long)
+    # The units split along the keys (with a workspace) are the last query
+    # blocks of the last head: sample rows there too.
+    lo = max(0, n - 16 * 256)
+    g = torch.Generator().manual_seed(seed + 1)
+    tail = torch.unique(torch.cat([lo + torch.randperm(n - lo, generator=g)[:16],
+                                   torch.tensor(_sampled_rows(n, 0, seed))]))
     heads = torch.randperm(w.H, generator=torch.Generator().manual_seed(seed))[:n_heads]
     heads = sorted(set(heads.tolist()) | {w.H - 1})
     for h in heads:
         kh, vh = kc[:, h:h + 1].contiguous(), vc[:, h:h + 1].contiguous()
         qh = q[:, h:h + 1].contiguous()
-        ref = oracle.attention(qh, kh, vh, q_idx=idx[rows])
-        _check_attention(out[rows, h:h + 1], ref, w.dtype)
+        r = rows if h != w.H - 1 else torch.unique(torch.cat([rows, tail]))
+        ref = oracle.attention(qh, kh, vh, q_idx=idx[r])
+        for out in outs:
+            _check_attention(out[r, h:h + 1], ref, w.dtype)
 
 
 @pytest.mark.parametrize("it", [0, 2, 1])
