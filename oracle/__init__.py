@@ -57,6 +57,7 @@ def lib():
             "orc_cached_euler_f64": [c_p, c_p, c_p, c_p, c_int, c_int, c_d],
             "orc_cached_euler_f32": [c_p, c_p, c_p, c_p, c_int, c_int, c_f],
             "orc_sigmas": [c_int, c_d, c_p],
+            "orc_l1rel_accumulate": [c_p, c_p, c_p, c_int, c_int, c_d, c_p],
         }
         for name, args in sig.items():
             f = getattr(_lib, name)
@@ -199,3 +200,14 @@ def sigmas(T: int, shift: float = 1.0) -> torch.Tensor:
     out = torch.empty(T + 1, dtype=torch.float64)
     _check(lib().orc_sigmas(T, float(shift), out.data_ptr()))
     return out
+
+
+def l1rel_accumulate(vhat_old, v_fresh, pos, weight: float, stat) -> None:
+    """In place on fp64 stat [N]: App. B Eq. 7 for the refreshed tokens."""
+    assert stat.dtype == torch.float64 and stat.is_contiguous()
+    vo = vhat_old.contiguous().to(torch.float64)
+    vf = v_fresh.contiguous().to(torch.float64)
+    p = pos.contiguous().to(torch.int32)
+    N, C = vo.shape
+    _check(lib().orc_l1rel_accumulate(vo.data_ptr(), vf.data_ptr(), p.data_ptr(), N, C,
+                                      float(weight), stat.data_ptr()))

@@ -22,12 +22,16 @@
  *   orc_cached_euler_*   Sec. 2.4 Eq. 6 (cached Euler update), with the
  *                        velocity cache refreshed for active tokens.
  *   orc_sigmas           Sec. 2.1 noise schedule of the Euler solver (Eq. 2).
+ *   orc_l1rel_accumulate App. B Eq. 7, the per-token L1 relative change of the
+ *                        velocity, accumulated (weighted) into a running mean.
  *
  * Readings where the paper is silent (each is listed with its reason in the
  * design notes): ties in the ranking go to the lower token index first and
  * -0 equals +0; a non-finite statistic is an error; the window margin is the
  * integer floor((100-k)*T/200) with k in percent; the softmax scale defaults
- * to 1/sqrt(D) with no mask; group ids are 0-based, group 0 the baseline.
+ * to 1/sqrt(D) with no mask; group ids are 0-based, group 0 the baseline; an
+ * L1 relative change with a zero denominator is 0 when the numerator is 0 and
+ * the largest finite fp32 value otherwise.
  *
  * Status codes (plain ints): 0 ok, -1 invalid argument, -2 a budget does not
  * divide T, -3 counts do not sum to N, -5 non-finite statistic, -6 index
@@ -358,6 +362,37 @@ int orc_sigmas(int T, double shift, double *sigma)
     for (int i = 0; i <= T; ++i) {
         double t = 1.0 - (double)i / (double)T;
         sigma[i] = shift * t / (1.0 + (shift - 1.0) * t);
+    }
+    return ORC_OK;
+}
+
+/* ------------------------------------------------- velocity statistic (D) */
+
+/* App. B Eq. 7: for every token refreshed at this step (pos[n] >= 0),
+ *   L1rel(n, i) = ||v_i[n] - v_{i-1}[n]||_1 / ||v_i[n]||_1
+ * with v_i[n] = v_fresh[pos[n]] and v_{i-1}[n] = vhat_old[n] (the velocity
+ * cache before this step's refresh), and stat[n] += weight * L1rel(n, i).
+ * With weight = 1/(number of averaged steps) stat ends as the mean over the
+ * initial full-budget steps, the statistic the dynamic selection ranks. */
+int orc_l1rel_accumulate(const double *vhat_old, const double *v_fresh, const int32_t *pos,
+                         int N, int C, double weight, double *stat)
+{
+    for (int n = 0; n < N; ++n) {
+        if (!pos || pos[n] < 0)
+            continue;
+        const double *vn = v_fresh + (size_t)pos[n] * C;
+        const double *vo = vhat_old + (size_t)n * C;
+        double num = 0.0, den = 0.0;
+        for (int c = 0; c < C; ++c) {
+            num += fabs(vn[c] - vo[c]);
+            den += fabs(vn[c]);
+        }
+        double r;
+        if (den == 0.0)
+            r = (num == 0.0) ? 0.0 : 3.4028234663852886e38;
+        else
+            r = num / den;
+        stat[n] += weight * r;
     }
     return ORC_OK;
 }

@@ -426,3 +426,43 @@ def test_euler_f32_mirror_within_rounding_bound():
     bound = 2 * T * 2.0 ** -24 * (x0.double().abs() + sum(v.double().abs() for v in vs) * 0.1)
     assert torch.all((x32.double() - x64).abs() <= bound)
     assert not torch.equal(x32.double(), x64)     # the mirror really is fp32
+
+
+# ------------------------------------------------- velocity statistic (D)
+
+def test_l1rel_closed_forms():
+    """App. B Eq. 7 on cases with known values: a velocity that doubles has
+    relative change 1/2, one that flips sign 2, one that stays 0; the measure
+    is scale invariant; skipped tokens are not touched."""
+    N, C = 6, 16
+    vo = synth.normal((N, C), 1).double()
+    vf = torch.stack([2 * vo[0], -vo[1], vo[2], 3.0 * vo[3], 7.5 * vo[4], vo[5]])
+    pos = torch.tensor([0, 1, 2, 3, 4, -1], dtype=torch.int32)
+    stat = torch.zeros(N, dtype=torch.float64)
+    oracle.l1rel_accumulate(vo, vf[:5].contiguous(), pos, 1.0, stat)
+    assert abs(stat[0] - 0.5) < 1e-15 and abs(stat[1] - 2.0) < 1e-15 and stat[2] == 0.0
+    assert abs(stat[3] - 2.0 / 3.0) < 1e-15 and abs(stat[4] - 6.5 / 7.5) < 1e-15
+    assert stat[5] == 0.0
+    s2 = torch.zeros(N, dtype=torch.float64)
+    oracle.l1rel_accumulate(4.0 * vo, 4.0 * vf[:5].contiguous(), pos, 1.0, s2)
+    assert torch.allclose(s2, stat, rtol=1e-14, atol=0)
+
+
+def test_l1rel_running_mean_and_zero_denominator():
+    N, C, steps = 40, 8, 9
+    g = torch.Generator().manual_seed(3)
+    vs = [torch.randn(N, C, generator=g, dtype=torch.float64) for _ in range(steps + 1)]
+    pos = torch.arange(N, dtype=torch.int32)
+    stat = torch.zeros(N, dtype=torch.float64)
+    for i in range(1, steps + 1):
+        oracle.l1rel_accumulate(vs[i - 1], vs[i], pos, 1.0 / steps, stat)
+    # the mean of the per-step relative changes, token by token
+    direct = sum(((vs[i] - vs[i - 1]).abs().sum(1) / vs[i].abs().sum(1))
+                 for i in range(1, steps + 1)) / steps
+    assert torch.allclose(stat, direct, rtol=1e-13)
+    z = torch.zeros(2, C, dtype=torch.float64)
+    s0 = torch.zeros(2, dtype=torch.float64)
+    one = torch.zeros(2, C, dtype=torch.float64)
+    one[1, 0] = 1.0
+    oracle.l1rel_accumulate(one, z, torch.tensor([0, 1], dtype=torch.int32), 1.0, s0)
+    assert s0[0] == 0.0 and s0[1] == 3.4028234663852886e38
