@@ -548,6 +548,19 @@ def memory_sweep():
             nbytes = (N - n) * 12 * C + n * 16 * C + 4 * N
             report("cached_euler", f"N={N} C={C}, half active", nbytes, ms)
             del x, vh, vfr, pos
+    for C in (16, 128):
+        for N in (1 << 20, 1 << 22, 1 << 24):
+            if N * C * 4 > (1 << 31):
+                continue
+            x = torch.empty((N, C), device=dev).normal_()
+            vh = torch.empty_like(x).normal_()
+            vfr = torch.empty_like(x).normal_()
+            pos = torch.arange(N, dtype=torch.int32, device=dev)
+            stat = torch.zeros(N, device=dev)
+            ms = timed(lambda: hsa.hsa_cached_euler_l1rel(x, vh, vfr, pos, -0.025, stat,
+                                                          1.0 / 9, N, stream))
+            report("cached_euler_l1rel", f"N={N} C={C}, all active", N * (20 * C + 12), ms)
+            del x, vh, vfr, pos, stat
     assert hsa.hsa_get_device_error(stream) == 0
 
 

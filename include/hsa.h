@@ -239,6 +239,20 @@ int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
                      const int32_t *pos, int n_fresh, int N, int C, float dsigma,
                      hsa_stream_t stream);
 
+/* Cached Euler update fused with the velocity statistic of the dynamic token
+ * selection (App. B, Eq. 7), for the initial full-budget iterations whose
+ * velocities rank the tokens.  For every token with pos[n] >= 0 it first adds
+ *   weight * ||v_fresh[pos[n]] - v_cache[n]||_1 / ||v_fresh[pos[n]]||_1
+ * to stat[n] (v_cache[n] still holds the previous step's velocity; a zero
+ * denominator adds 0 when the numerator is 0 and weight * FLT_MAX otherwise),
+ * then performs exactly hsa_cached_euler.  With weight = 1/(number of steps
+ * averaged) stat ends as the mean relative change, ready for hsa_partition.
+ *   stat  device, fp32 [N], accumulated in place (fp32 fma).
+ * pos and v_fresh are required; other arguments as for hsa_cached_euler. */
+int hsa_cached_euler_l1rel(float *x, float *v_cache, const float *v_fresh,
+                           const int32_t *pos, int n_fresh, int N, int C, float dsigma,
+                           float *stat, float weight, hsa_stream_t stream);
+
 /* ------------------------------------------------------------------ errors */
 
 /* Waits for `stream`, then reports and clears the device-side errors recorded

@@ -22,7 +22,7 @@ __all__ = [
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
     "hsa_partition", "hsa_partition_static", "hsa_partition_active", "hsa_gather_active",
     "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_active_attention_workspace_bytes",
-    "hsa_cached_euler",
+    "hsa_cached_euler", "hsa_cached_euler_l1rel",
     "hsa_get_device_error", "hsa_test_inject_attention_stall",
 ]
 
@@ -65,6 +65,8 @@ _SIGS = {
                               _c_p, _c_int, _c_p, _c_sz, _c_p], _c_int),
     "hsa_active_attention_workspace_bytes": ([_c_int, _c_int, _c_int, _c_int, _c_int], _c_sz),
     "hsa_cached_euler": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p], _c_int),
+    "hsa_cached_euler_l1rel": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p,
+                                _c_f, _c_p], _c_int),
     "hsa_get_device_error": ([_c_p], _c_int),
     "hsa_test_inject_attention_stall": ([_c_int], _c_int),
 }
@@ -230,6 +232,16 @@ def hsa_cached_euler(x, v_cache, v_fresh, pos, dsigma: float, n_fresh: int | Non
         n_fresh = 0 if v_fresh is None else v_fresh.shape[0]
     _check(lib().hsa_cached_euler(_p(x), _p(v_cache), _p(v_fresh), _p(pos), n_fresh, N, C,
                                   float(dsigma), _stream(stream)), "hsa_cached_euler")
+
+
+def hsa_cached_euler_l1rel(x, v_cache, v_fresh, pos, dsigma: float, stat, weight: float,
+                           n_fresh: int | None = None, stream=None) -> None:
+    N, C = x.shape
+    if n_fresh is None:
+        n_fresh = v_fresh.shape[0]
+    _check(lib().hsa_cached_euler_l1rel(_p(x), _p(v_cache), _p(v_fresh), _p(pos), n_fresh, N, C,
+                                        float(dsigma), _p(stat), float(weight),
+                                        _stream(stream)), "hsa_cached_euler_l1rel")
 
 
 def hsa_get_device_error(stream=None) -> int:

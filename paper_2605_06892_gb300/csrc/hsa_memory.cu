@@ -153,6 +153,92 @@ cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
   }
 }
 
+// Cached Euler step fused with the velocity statistic of the dynamic token
+// selection (App. B, Eq. 7): for a refreshed token (pos[n] >= 0) the old cache
+// row is v_{i-1}[n] and the fresh row v_i[n]; the kernel adds
+// weight * ||v_i - v_{i-1}||_1 / ||v_i||_1 to stat[n] (a zero denominator
+// counts 0 with a zero numerator, FLT_MAX otherwise), then refreshes the cache
+// and advances x exactly as cached_euler_kernel does.  A group of L lanes owns
+// a token; the two L1 norms are reduced across the group with shuffles.
+constexpr int kL1relRows = 2;   // tokens per lane group per pass
+
+__global__ void __launch_bounds__(kThreads, 4)
+euler_l1rel_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
+                   const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
+                   int N, int vecs, int lpr_log2, float dsigma, int n_fresh_rows,
+                   float *__restrict__ stat, float weight, unsigned *err) {
+  const int L = 1 << lpr_log2;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> lpr_log2;
+  const int sl = lane & (L - 1);
+  const int rows_per_warp = 32 >> lpr_log2;
+  const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+  const long long step = nwarps * rows_per_warp;            // between a group's tokens
+  // All lanes of a warp run the same number of passes (the shuffles below
+  // span the warp): the bound is the token count rounded up to whole passes.
+  const long long span = step * kL1relRows;
+  const long long rows_pad = ((long long)N + span - 1) / span * span;
+  for (long long n0 = warp * rows_per_warp; n0 < rows_pad; n0 += span) {
+    long long n[kL1relRows];
+    int p[kL1relRows];
+#pragma unroll
+    for (int k = 0; k < kL1relRows; ++k) {
+      n[k] = n0 + k * step + sub;
+      p[k] = (n[k] < N) ? __ldg(pos + n[k]) : -1;
+      if (p[k] >= n_fresh_rows) {
+        set_error(err, kErrIndex);
+        p[k] = -1;
+      }
+    }
+    float num[kL1relRows], den[kL1relRows];
+#pragma unroll
+    for (int k = 0; k < kL1relRows; ++k) num[k] = den[k] = 0.f;
+    for (int v = sl; v < vecs; v += L) {
+      float4 vo[kL1relRows], vn[kL1relRows], xv[kL1relRows];
+#pragma unroll
+      for (int k = 0; k < kL1relRows; ++k) {
+        if (n[k] < N) {
+          vo[k] = vhat[n[k] * vecs + v];
+          vn[k] = p[k] >= 0 ? __ldg(v_fresh + (long long)p[k] * vecs + v) : vo[k];
+          xv[k] = x[n[k] * vecs + v];
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < kL1relRows; ++k) {
+        if (n[k] < N) {
+          if (p[k] >= 0) {
+            num[k] += fabsf(vn[k].x - vo[k].x) + fabsf(vn[k].y - vo[k].y) +
+                      fabsf(vn[k].z - vo[k].z) + fabsf(vn[k].w - vo[k].w);
+            den[k] += fabsf(vn[k].x) + fabsf(vn[k].y) + fabsf(vn[k].z) + fabsf(vn[k].w);
+            vhat[n[k] * vecs + v] = vn[k];
+          }
+          float4 o;
+          o.x = __fmaf_rn(vn[k].x, dsigma, xv[k].x);
+          o.y = __fmaf_rn(vn[k].y, dsigma, xv[k].y);
+          o.z = __fmaf_rn(vn[k].z, dsigma, xv[k].z);
+          o.w = __fmaf_rn(vn[k].w, dsigma, xv[k].w);
+          x[n[k] * vecs + v] = o;
+        }
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kL1relRows; ++k) {
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        if (o < L) {
+          num[k] += __shfl_xor_sync(0xffffffffu, num[k], o);
+          den[k] += __shfl_xor_sync(0xffffffffu, den[k], o);
+        }
+      }
+      if (n[k] < N && p[k] >= 0 && sl == 0) {
+        const float r = den[k] > 0.f ? num[k] / den[k] : (num[k] > 0.f ? 3.402823466e38f : 0.f);
+        stat[n[k]] = fmaf(weight, r, stat[n[k]]);
+      }
+    }
+  }
+}
+
 // Grid for n_rows rows handled by lane groups of size L: up to 8 blocks of
 // 256 threads per SM (a full SM), no more than the rows need; blocks beyond
 // what is resident wait their turn.
@@ -242,5 +328,25 @@ extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
     cached_euler_kernel<1><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
         (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
         dsigma, pos ? n_fresh : 0, err);
+  return launch_status();
+}
+
+extern "C" int hsa_cached_euler_l1rel(float *x, float *v_cache, const float *v_fresh,
+                                      const int32_t *pos, int n_fresh, int N, int C,
+                                      float dsigma, float *stat, float weight,
+                                      hsa_stream_t stream) {
+  if (N < 0 || C < 4 || (C & 3) || n_fresh < 0) return HSA_ERR_INVALID_ARG;
+  if (!pos || !v_fresh || !stat) return HSA_ERR_INVALID_ARG;
+  if (N == 0) return HSA_OK;
+  if (!x || !v_cache || !aligned16(x) || !aligned16(v_cache) || !aligned16(v_fresh))
+    return HSA_ERR_INVALID_ARG;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const int vecs = C / 4;
+  const int L = lanes_per_row(vecs);
+  euler_l1rel_kernel<<<grid_for(((long long)N + kL1relRows - 1) / kL1relRows, L), kThreads, 0,
+                       (cudaStream_t)stream>>>(
+      (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, N, vecs, log2i(L), dsigma,
+      n_fresh, stat, weight, err);
   return launch_status();
 }
