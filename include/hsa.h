@@ -142,6 +142,21 @@ int hsa_partition_static(const float *stat, int N, int T, const int *budgets,
                          const int *counts, int K, int32_t *group_of,
                          hsa_stream_t stream);
 
+/* Statistics for the other token allocation strategies of App. B, to be
+ * ranked by hsa_partition (the random strategy R ranks any random statistic
+ * the caller draws):
+ *  - uniform allocation (U): stat[n] = top 24 bits of (n+1) * 2654435769 mod
+ *    2^32 (golden-ratio sequence), an exact integer in fp32.  Each group then
+ *    holds the tokens of one interval of the sequence, which are spaced by at
+ *    most three distinct gaps over the whole token range ("maximally spread").
+ *  - first-frame reservation (F): stat[n] = FLT_MAX for n < frame_tokens (the
+ *    first latent frame, (H_l/2)*(W_l/2) tokens in row-major order), applied
+ *    on top of a random statistic; with counts[0] >= frame_tokens every
+ *    first-frame token lands in the baseline group.
+ *   stat  device, fp32 [N], written (U) or updated in place (F). */
+int hsa_uniform_stat(float *stat, int N, hsa_stream_t stream);
+int hsa_reserve_first_frame(float *stat, int N, int frame_tokens, hsa_stream_t stream);
+
 /* ---------------------------------------------------- a2 active set per step */
 
 /* Active set A_i (Sec. 2.3; Fig. 1): token n is active at iteration iter iff

@@ -58,6 +58,8 @@ def lib():
             "orc_cached_euler_f32": [c_p, c_p, c_p, c_p, c_int, c_int, c_f],
             "orc_sigmas": [c_int, c_d, c_p],
             "orc_l1rel_accumulate": [c_p, c_p, c_p, c_int, c_int, c_d, c_p],
+            "orc_uniform_stat": [c_int, c_p],
+            "orc_reserve_frame": [c_p, c_int, c_int],
         }
         for name, args in sig.items():
             f = getattr(_lib, name)
@@ -211,3 +213,15 @@ def l1rel_accumulate(vhat_old, v_fresh, pos, weight: float, stat) -> None:
     N, C = vo.shape
     _check(lib().orc_l1rel_accumulate(vo.data_ptr(), vf.data_ptr(), p.data_ptr(), N, C,
                                       float(weight), stat.data_ptr()))
+
+
+def uniform_stat(N: int) -> torch.Tensor:
+    out = torch.empty(max(N, 1), dtype=torch.float32)
+    _check(lib().orc_uniform_stat(N, out.data_ptr()))
+    return out[:N].clone()
+
+
+def reserve_frame(stat: torch.Tensor, frame_tokens: int) -> torch.Tensor:
+    out = stat.contiguous().to(torch.float32).clone()
+    _check(lib().orc_reserve_frame(out.data_ptr(), out.numel(), frame_tokens))
+    return out

@@ -24,6 +24,9 @@
  *   orc_sigmas           Sec. 2.1 noise schedule of the Euler solver (Eq. 2).
  *   orc_l1rel_accumulate App. B Eq. 7, the per-token L1 relative change of the
  *                        velocity, accumulated (weighted) into a running mean.
+ *   orc_uniform_stat     App. B "uniform allocation (U)": a statistic whose
+ *                        ranking gives every group evenly spread positions.
+ *   orc_reserve_frame    App. B "first-frame reservation (F)".
  *
  * Readings where the paper is silent (each is listed with its reason in the
  * design notes): ties in the ranking go to the lower token index first and
@@ -394,5 +397,34 @@ int orc_l1rel_accumulate(const double *vhat_old, const double *v_fresh, const in
             r = num / den;
         stat[n] += weight * r;
     }
+    return ORC_OK;
+}
+
+/* -------------------------------------------------- allocation strategies */
+
+/* Uniform allocation (App. B, U).  Reading: token n gets the statistic
+ * floor(frac((n+1) * phi) * 2^24) with phi = (sqrt(5)-1)/2, taken as the top
+ * 24 bits of the 32-bit product (n+1) * 2654435769 (= round(phi * 2^32)).
+ * Ranking it (orc_partition) gives each group the tokens whose value lies in
+ * one interval of the circle, which by the three-distance theorem are spaced
+ * by at most three distinct gaps: maximally spread over the sequence. */
+int orc_uniform_stat(int N, float *stat)
+{
+    for (int n = 0; n < N; ++n) {
+        uint32_t h = (uint32_t)(n + 1) * 2654435769u;
+        stat[n] = (float)(h >> 8);
+    }
+    return ORC_OK;
+}
+
+/* First-frame reservation (App. B, F): the first frame_tokens tokens (frame 0
+ * in row-major token order) get the largest finite fp32 statistic, so a
+ * ranking places them in the baseline group when |G_1| >= frame_tokens. */
+int orc_reserve_frame(float *stat, int N, int frame_tokens)
+{
+    if (frame_tokens < 0 || frame_tokens > N)
+        return ORC_EINVAL;
+    for (int n = 0; n < frame_tokens; ++n)
+        stat[n] = 3.40282347e38f;
     return ORC_OK;
 }

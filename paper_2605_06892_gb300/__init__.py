@@ -20,7 +20,8 @@ __all__ = [
     "HsaError", "lib", "library_path", "HSA_BF16", "HSA_F32",
     "hsa_status_string", "hsa_version", "hsa_check_budgets", "hsa_window_margin",
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
-    "hsa_partition", "hsa_partition_static", "hsa_partition_active", "hsa_gather_active",
+    "hsa_partition", "hsa_partition_static", "hsa_uniform_stat", "hsa_reserve_first_frame",
+    "hsa_partition_active", "hsa_gather_active",
     "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_active_attention_workspace_bytes",
     "hsa_cached_euler", "hsa_cached_euler_l1rel",
     "hsa_get_device_error", "hsa_test_inject_attention_stall",
@@ -56,6 +57,8 @@ _SIGS = {
     "hsa_partition": ([_c_p, _c_int, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p, _c_sz, _c_p],
                       _c_int),
     "hsa_partition_static": ([_c_p, _c_int, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p], _c_int),
+    "hsa_uniform_stat": ([_c_p, _c_int, _c_p], _c_int),
+    "hsa_reserve_first_frame": ([_c_p, _c_int, _c_int, _c_p], _c_int),
     "hsa_partition_active": ([_c_p, _c_int, _c_int, _c_p, _c_int, _c_int, _c_int, _c_p, _c_p,
                               _c_p], _c_int),
     "hsa_gather_active": ([_c_p, _c_sz, _c_int, _c_p, _c_int, _c_p, _c_p], _c_int),
@@ -182,6 +185,17 @@ def hsa_partition_static(stat, T: int, budgets, counts, group_of, stream=None) -
     _check(lib().hsa_partition_static(_p(stat), stat.numel(), T, _host_ints(budgets),
                                       _host_ints(counts), len(budgets), _p(group_of),
                                       _stream(stream)), "hsa_partition_static")
+
+
+def hsa_uniform_stat(stat, stream=None) -> None:
+    """stat[n] <- uniform-allocation statistic (App. B, U)."""
+    _check(lib().hsa_uniform_stat(_p(stat), stat.numel(), _stream(stream)), "hsa_uniform_stat")
+
+
+def hsa_reserve_first_frame(stat, frame_tokens: int, stream=None) -> None:
+    """stat[:frame_tokens] <- FLT_MAX (App. B, F)."""
+    _check(lib().hsa_reserve_first_frame(_p(stat), stat.numel(), frame_tokens,
+                                         _stream(stream)), "hsa_reserve_first_frame")
 
 
 def hsa_partition_active(group_of, T: int, budgets, iter_: int, idx, pos=None,

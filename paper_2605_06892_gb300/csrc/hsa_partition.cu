@@ -338,6 +338,27 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
   return launch_status();
 }
 
+// ------------------------------------------------- allocation strategies
+//
+// Statistics whose ranking by hsa_partition gives the other token allocation
+// strategies of App. B.  Uniform (U): stat[n] = top 24 bits of the 32-bit
+// product (n+1) * 2654435769 (the golden ratio times 2^32), an integer exactly
+// representable in fp32; each group then takes the tokens of one interval of
+// the golden-ratio sequence, spaced by at most three distinct gaps.
+// First-frame reservation (F): the first frame's tokens get FLT_MAX, so they
+// rank into the baseline group.
+
+__global__ void uniform_stat_kernel(float *__restrict__ stat, int N) {
+  for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < N; n += gridDim.x * blockDim.x)
+    stat[n] = (float)(((uint32_t)(n + 1) * 2654435769u) >> 8);
+}
+
+__global__ void reserve_frame_kernel(float *__restrict__ stat, int frame_tokens) {
+  for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < frame_tokens;
+       n += gridDim.x * blockDim.x)
+    stat[n] = 3.40282347e38f;
+}
+
 // ----------------------------------------------- partition without allocation
 //
 // Variant of hsa_partition for callers that cannot hand the library a
@@ -386,4 +407,23 @@ extern "C" int hsa_partition_static(const float *stat, int N, int T, const int *
   if (!scratch) return HSA_ERR_CUDA;
   return hsa_partition(stat, N, T, budgets, counts, K, group_of, scratch, kStaticScratchBytes,
                        stream);
+}
+
+extern "C" int hsa_uniform_stat(float *stat, int N, hsa_stream_t stream) {
+  if (N < 0) return HSA_ERR_INVALID_ARG;
+  if (N == 0) return HSA_OK;
+  if (!stat) return HSA_ERR_INVALID_ARG;
+  const int blocks = (int)std::min<long long>((N + 255) / 256, (long long)sm_count() * 8);
+  uniform_stat_kernel<<<blocks, 256, 0, (cudaStream_t)stream>>>(stat, N);
+  return launch_status();
+}
+
+extern "C" int hsa_reserve_first_frame(float *stat, int N, int frame_tokens,
+                                       hsa_stream_t stream) {
+  if (N < 0 || frame_tokens < 0 || frame_tokens > N) return HSA_ERR_INVALID_ARG;
+  if (frame_tokens == 0) return HSA_OK;
+  if (!stat) return HSA_ERR_INVALID_ARG;
+  const int blocks = (int)std::min<long long>((frame_tokens + 255) / 256, (long long)sm_count() * 8);
+  reserve_frame_kernel<<<blocks, 256, 0, (cudaStream_t)stream>>>(stat, frame_tokens);
+  return launch_status();
 }

@@ -111,6 +111,31 @@ def test_partition_errors(hsa):
     _no_device_error(hsa)
 
 
+@pytest.mark.parametrize("name", ["wan13b", "ltx", "wan14b_720p", "tiny_f32"])
+def test_allocation_strategies_u_and_f(hsa, name):
+    """U and F statistics match the oracle bit for bit and give the same
+    partitions (App. B)."""
+    w = synth.WORKLOADS[name]
+    counts = w.counts
+    st = torch.empty(w.N, device=DEV)
+    hsa.hsa_uniform_stat(st)
+    ref = oracle.uniform_stat(w.N)
+    assert torch.equal(st.cpu(), ref)
+    assert torch.equal(_gpu_partition(hsa, st.cpu(), w.T, w.budgets, counts),
+                       oracle.partition(ref, w.T, w.budgets, counts))
+    frame = w.grid[1] * w.grid[2]
+    if counts[0] >= frame:
+        rnd = torch.rand(w.N, generator=torch.Generator().manual_seed(w.cid))
+        st = rnd.to(DEV)
+        hsa.hsa_reserve_first_frame(st, frame)
+        ref_f = oracle.reserve_frame(rnd, frame)
+        assert torch.equal(st.cpu(), ref_f)
+        g = _gpu_partition(hsa, st.cpu(), w.T, w.budgets, counts)
+        assert torch.equal(g, oracle.partition(ref_f, w.T, w.budgets, counts))
+        assert torch.all(g[:frame] == 0)
+    _no_device_error(hsa)
+
+
 # -------------------------------------------------------------- active set
 
 @pytest.mark.parametrize("name", list(synth.WORKLOADS))

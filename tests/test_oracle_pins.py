@@ -466,3 +466,45 @@ def test_l1rel_running_mean_and_zero_denominator():
     one[1, 0] = 1.0
     oracle.l1rel_accumulate(one, z, torch.tensor([0, 1], dtype=torch.int32), 1.0, s0)
     assert s0[0] == 0.0 and s0[1] == 3.4028234663852886e38
+
+
+# ---------------------------------------------------- allocation strategies
+
+@pytest.mark.parametrize("name", ["wan13b", "ltx", "wan14b_720p"])
+def test_uniform_allocation_three_gaps(name):
+    """U: each group's members are spaced by at most three distinct gaps
+    (three-distance theorem) whose mean is N/|G_k|, and every group reaches
+    both ends of the sequence."""
+    w = synth.WORKLOADS[name]
+    stat = oracle.uniform_stat(w.N)
+    # the statistic is a permutation-free set of distinct values here
+    assert torch.unique(stat).numel() == w.N
+    g = oracle.partition(stat, w.T, w.budgets, w.counts)
+    for k, c in enumerate(w.counts):
+        members = torch.nonzero(g == k).flatten()
+        assert members.numel() == c
+        gaps = torch.unique(members[1:] - members[:-1])
+        assert gaps.numel() <= 3, gaps
+        assert members[0] < 2 * w.N / c and members[-1] > w.N - 2 * w.N / c
+        assert abs(float((members[1:] - members[:-1]).double().mean()) - w.N / c) < 0.01 * w.N / c + 1
+
+
+def test_uniform_stat_closed_form():
+    s = oracle.uniform_stat(5)
+    phi = (5 ** 0.5 - 1) / 2
+    for n in range(5):
+        assert s[n] == math.floor(((n + 1) * phi % 1.0) * 2 ** 24) or \
+            abs(float(s[n]) - ((n + 1) * phi % 1.0) * 2 ** 24) <= 1.0
+
+
+def test_first_frame_reservation():
+    """F: with |G_1| >= frame size, every token of frame 0 is in the baseline
+    group; the rest are ranked by the (random) statistic."""
+    w = synth.WORKLOADS["wan13b"]
+    frame = w.grid[1] * w.grid[2]
+    stat = torch.rand(w.N, generator=torch.Generator().manual_seed(9))
+    g = oracle.partition(oracle.reserve_frame(stat, frame), w.T, w.budgets, w.counts)
+    assert torch.all(g[:frame] == 0)
+    rest = oracle.partition(stat[frame:].contiguous(), w.T, w.budgets,
+                            (w.counts[0] - frame,) + tuple(w.counts[1:]))
+    assert torch.equal(g[frame:], rest)
