@@ -60,6 +60,7 @@ def lib():
             "orc_l1rel_accumulate": [c_p, c_p, c_p, c_int, c_int, c_d, c_p],
             "orc_uniform_stat": [c_int, c_p],
             "orc_reserve_frame": [c_p, c_int, c_int],
+            "orc_reorder": [c_p, c_int, c_p, c_p, c_p],
         }
         for name, args in sig.items():
             f = getattr(_lib, name)
@@ -225,3 +226,13 @@ def reserve_frame(stat: torch.Tensor, frame_tokens: int) -> torch.Tensor:
     out = stat.contiguous().to(torch.float32).clone()
     _check(lib().orc_reserve_frame(out.data_ptr(), out.numel(), frame_tokens))
     return out
+
+
+def reorder(group_of: torch.Tensor):
+    """(order, where, group_new, M) of the Sec. 2.5 token reordering."""
+    g = group_of.contiguous().to(torch.int32)
+    N = g.numel()
+    order, where, gn = (torch.empty(max(N, 1), dtype=torch.int32) for _ in range(3))
+    M = _check(lib().orc_reorder(g.data_ptr(), N, order.data_ptr(), where.data_ptr(),
+                                 gn.data_ptr()))
+    return order[:N].clone(), where[:N].clone(), gn[:N].clone(), M

@@ -27,6 +27,8 @@
  *   orc_uniform_stat     App. B "uniform allocation (U)": a statistic whose
  *                        ranking gives every group evenly spread positions.
  *   orc_reserve_frame    App. B "first-frame reservation (F)".
+ *   orc_reorder          Sec. 2.5 "token reordering": non-baseline tokens
+ *                        first, then the baseline group, each in token order.
  *
  * Readings where the paper is silent (each is listed with its reason in the
  * design notes): ties in the ranking go to the lower token index first and
@@ -427,4 +429,34 @@ int orc_reserve_frame(float *stat, int N, int frame_tokens)
     for (int n = 0; n < frame_tokens; ++n)
         stat[n] = 3.40282347e38f;
     return ORC_OK;
+}
+
+/* ------------------------------------------------------- token reordering */
+
+/* Token reordering (Sec. 2.5): new position r holds old token order[r]; the
+ * tokens of groups 1..K-1 come first in their original order, then the
+ * baseline group 0 in its original order.  where[n] is the new position of
+ * old token n (the inverse permutation, used to undo the reordering), and
+ * group_new[r] = group_of[order[r]].  Returns the number of non-baseline
+ * tokens M (the length of the cached prefix). */
+int orc_reorder(const int32_t *group_of, int N, int32_t *order, int32_t *where,
+                int32_t *group_new)
+{
+    int r = 0;
+    for (int n = 0; n < N; ++n)
+        if (group_of[n] != 0) {
+            order[r] = n;
+            where[n] = r;
+            group_new[r] = group_of[n];
+            ++r;
+        }
+    const int M = r;
+    for (int n = 0; n < N; ++n)
+        if (group_of[n] == 0) {
+            order[r] = n;
+            where[n] = r;
+            group_new[r] = 0;
+            ++r;
+        }
+    return M;
 }

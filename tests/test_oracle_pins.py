@@ -508,3 +508,57 @@ def test_first_frame_reservation():
     rest = oracle.partition(stat[frame:].contiguous(), w.T, w.budgets,
                             (w.counts[0] - frame,) + tuple(w.counts[1:]))
     assert torch.equal(g[frame:], rest)
+
+
+# --------------------------------------------------------- token reordering
+
+def test_reorder_is_stable_partition_with_inverse():
+    w = synth.WORKLOADS["ltx"]
+    stat, counts = synth.stat_for(w)
+    g = oracle.partition(stat, w.T, w.budgets, counts)
+    order, where, gn, M = oracle.reorder(g)
+    N = w.N
+    assert M == N - counts[0]
+    assert torch.equal(torch.sort(order).values, torch.arange(N, dtype=torch.int32))
+    assert torch.equal(where[order.long()], torch.arange(N, dtype=torch.int32))
+    assert torch.all(gn[:M] != 0) and torch.all(gn[M:] == 0)
+    assert torch.equal(gn, g[order.long()])
+    assert torch.all(order[1:M] > order[:M - 1]) and torch.all(order[M + 1:] > order[M:-1])
+
+
+def test_reordered_cache_gives_the_same_attention():
+    """Sec. 2.5: the baseline group is active at every iteration, so a cache
+    over the non-baseline prefix plus the fresh baseline K/V holds exactly the
+    keys of the full cache.  Over a T = 8 schedule, attention outputs with the
+    reordered, prefix-only cache equal (permuted back) those with the full
+    cache."""
+    N, H, D, T = 90, 2, 16, 8
+    budgets, counts = (8, 4, 2), (20, 30, 40)
+    g = oracle.partition(torch.rand(N, generator=torch.Generator().manual_seed(3)), T,
+                         budgets, counts)
+    order, where, gn, M = oracle.reorder(g)
+    kc_full = synth.normal((N, H, D), 1)
+    vc_full = synth.normal((N, H, D), 2)
+    kc_pre = kc_full[order[:M].long()].contiguous()
+    vc_pre = vc_full[order[:M].long()].contiguous()
+    for it in range(T):
+        kf = synth.normal((N, H, D), 100 + it)        # fresh K/V of every token
+        vf = synth.normal((N, H, D), 200 + it)
+        q = synth.normal((N, H, D), 300 + it)
+        idx, _ = oracle.active_set(g, T, budgets, it)
+        oracle.kv_scatter(kc_full, vc_full, kf[idx.long()].contiguous(),
+                          vf[idx.long()].contiguous(), idx)
+        ref = oracle.attention(q, kc_full, vc_full, q_idx=idx)
+        idx_new, _ = oracle.active_set(gn, T, budgets, it)
+        nb = int((idx_new < M).sum())
+        assert torch.equal(idx_new[nb:], torch.arange(M, N, dtype=torch.int32))
+        old_of_new = order[idx_new.long()].long()
+        oracle.kv_scatter(kc_pre, vc_pre, kf[old_of_new[:nb]].contiguous(),
+                          vf[old_of_new[:nb]].contiguous(), idx_new[:nb].contiguous())
+        kb, vb = kf[order[M:].long()], vf[order[M:].long()]   # fresh baseline K/V
+        got = oracle.attention(q[old_of_new].contiguous(), torch.cat([kc_pre, kb]).contiguous(),
+                               torch.cat([vc_pre, vb]).contiguous())
+        # rows of A_i in new order vs old order: same tokens
+        assert torch.equal(torch.sort(old_of_new).values.to(torch.int32), idx)
+        perm = torch.argsort(old_of_new)
+        assert torch.allclose(got[perm], ref, atol=1e-12)
