@@ -157,6 +157,22 @@ int hsa_partition_static(const float *stat, int N, int T, const int *budgets,
 int hsa_uniform_stat(float *stat, int N, hsa_stream_t stream);
 int hsa_reserve_first_frame(float *stat, int N, int frame_tokens, hsa_stream_t stream);
 
+/* Token reordering (Sec. 2.5), applied once before the denoising loop: new
+ * position r holds old token order[r]; the tokens of groups 1..K-1 come first
+ * in token order, then the n_baseline tokens of the baseline group (group 0),
+ * also in token order.  The KV cache then only needs the prefix of
+ * M = N - n_baseline rows, because the baseline group is active at every
+ * iteration (see hsa_active_attention_prefix).
+ *   group_of   device, int32 [N]; exactly n_baseline entries are 0.
+ *   order      device, int32 [N], written (new -> old).  Reorder a per-token
+ *              tensor with hsa_gather_active(src, .., order, N, dst).
+ *   where      device, int32 [N] or NULL, written (old -> new); undo the
+ *              reordering with hsa_gather_active(.., where, N, ..).
+ *   group_new  device, int32 [N] or NULL, written: group_of[order[r]].
+ * A group_of that disagrees with n_baseline is reported as HSA_ERR_INDEX. */
+int hsa_reorder_tokens(const int32_t *group_of, int N, int n_baseline, int32_t *order,
+                       int32_t *where, int32_t *group_new, hsa_stream_t stream);
+
 /* ---------------------------------------------------- a2 active set per step */
 
 /* Active set A_i (Sec. 2.3; Fig. 1): token n is active at iteration iter iff
@@ -230,6 +246,19 @@ int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
                          int D, float scale, void *out, hsa_dtype dtype,
                          void *workspace, size_t workspace_bytes,
                          hsa_stream_t stream);
+
+/* hsa_active_attention over keys held in two sources, read in order: the M
+ * rows of k_cache / v_cache ([M, H, D], the cache of the non-baseline prefix
+ * after token reordering, Sec. 2.5) followed by the B rows of k_base /
+ * v_base ([B, H, D], the fresh K/V of the baseline group, which is active at
+ * every iteration).  Keys total M + B >= 1; either source may be empty.
+ * q_idx, when given, indexes a [M + B, H, D] query tensor.  Everything else
+ * as hsa_active_attention (which is this call with B = 0). */
+int hsa_active_attention_prefix(const void *q, const int32_t *q_idx, int n_active,
+                                const void *k_cache, const void *v_cache, int M,
+                                const void *k_base, const void *v_base, int B, int H, int D,
+                                float scale, void *out, hsa_dtype dtype, void *workspace,
+                                size_t workspace_bytes, hsa_stream_t stream);
 
 /* Workspace bytes that let hsa_active_attention balance its last wave (0 when
  * the dtype or shape takes none).  Depends only on the device's SM count and

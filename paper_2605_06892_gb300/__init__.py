@@ -21,8 +21,9 @@ __all__ = [
     "hsa_status_string", "hsa_version", "hsa_check_budgets", "hsa_window_margin",
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
     "hsa_partition", "hsa_partition_static", "hsa_uniform_stat", "hsa_reserve_first_frame",
-    "hsa_partition_active", "hsa_gather_active",
-    "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_active_attention_workspace_bytes",
+    "hsa_reorder_tokens", "hsa_partition_active", "hsa_gather_active",
+    "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_active_attention_prefix",
+    "hsa_active_attention_workspace_bytes",
     "hsa_cached_euler", "hsa_cached_euler_l1rel",
     "hsa_get_device_error", "hsa_test_inject_attention_stall",
 ]
@@ -66,6 +67,10 @@ _SIGS = {
                              _c_int, _c_p], _c_int),
     "hsa_active_attention": ([_c_p, _c_p, _c_int, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f,
                               _c_p, _c_int, _c_p, _c_sz, _c_p], _c_int),
+    "hsa_active_attention_prefix": ([_c_p, _c_p, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p, _c_int,
+                                     _c_int, _c_int, _c_f, _c_p, _c_int, _c_p, _c_sz, _c_p],
+                                    _c_int),
+    "hsa_reorder_tokens": ([_c_p, _c_int, _c_int, _c_p, _c_p, _c_p, _c_p], _c_int),
     "hsa_active_attention_workspace_bytes": ([_c_int, _c_int, _c_int, _c_int, _c_int], _c_sz),
     "hsa_cached_euler": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p], _c_int),
     "hsa_cached_euler_l1rel": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p,
@@ -219,6 +224,26 @@ def hsa_kv_sync_scatter(k_cache, v_cache, k_fresh, v_fresh, idx, n_active: int,
     _check(lib().hsa_kv_sync_scatter(_p(k_cache), _p(v_cache), _p(k_fresh), _p(v_fresh),
                                      _p(idx), n_active, N, H, D, _dtype_code(k_cache),
                                      _stream(stream)), "hsa_kv_sync_scatter")
+
+
+def hsa_active_attention_prefix(q, q_idx, n_active: int, k_cache, v_cache, k_base, v_base, out,
+                                scale: float = 0.0, workspace=None, stream=None) -> None:
+    """Attention against the M cached rows followed by the B baseline rows."""
+    M, H, D = k_cache.shape
+    B = k_base.shape[0]
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().hsa_active_attention_prefix(
+        _p(q), _p(q_idx), n_active, _p(k_cache) if M else None, _p(v_cache) if M else None, M,
+        _p(k_base) if B else None, _p(v_base) if B else None, B, H, D, float(scale), _p(out),
+        _dtype_code(k_cache if M else k_base), _p(workspace), ws_bytes, _stream(stream)),
+        "hsa_active_attention_prefix")
+
+
+def hsa_reorder_tokens(group_of, n_baseline: int, order, where=None, group_new=None,
+                       stream=None) -> None:
+    _check(lib().hsa_reorder_tokens(_p(group_of), group_of.numel(), n_baseline, _p(order),
+                                    _p(where), _p(group_new), _stream(stream)),
+           "hsa_reorder_tokens")
 
 
 def hsa_active_attention_workspace_bytes(n_active: int, N: int, H: int, D: int,

@@ -2,8 +2,10 @@
 // queries attend to all N rows of the layer's KV cache, O(|A_i| N) work.
 //
 // bf16 path: one CTA owns 256 active query rows (two 128-row Q tiles) of one
-// head and streams every 128-key tile of that head's cache through shared
-// memory.  Warp roles:
+// head and streams every 128-key tile of that head's keys through shared
+// memory.  The keys are the rows of up to two sources read in order: the KV
+// cache, then (token reordering, Sec. 2.5) the fresh K/V of the baseline
+// group, which is active at every iteration and so needs no cache.  Warp roles:
 //   warp 0      TMA producer: K and V tiles of the head, 128-byte swizzled,
 //               into a ring of shared-memory slots (rows >= N are zero-filled).
 //   warp 1      tensor-core issuer (one thread): S_t = Q_t K^T into TMEM and
@@ -295,6 +297,7 @@ struct TcArgs {
   __nv_bfloat16 *out;
   unsigned *err;
   int n_active, N, H, q_rows, n_kv_tiles;
+  int rows1, rows2, tiles1;   // key sources: rows1 cache rows, then rows2 rows
   float scale_log2;
   int inject_stall;   // test hook (hsa_test.h): 1 = tile 0 withholds its first P
   // Work split.  CTA b < n_whole owns unit b (head b / n_qblocks, query block
@@ -412,6 +415,7 @@ __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid
 template <int D>
 __global__ void __launch_bounds__(kTcThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+               const __grid_constant__ CUtensorMap tm_k2, const __grid_constant__ CUtensorMap tm_v2,
                const TcArgs a) {
   using C = TcCfg<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -493,12 +497,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
           const int slot = L % C::kStages, use = L / C::kStages;
           if (use > 0 && !mbar_wait(&bar_empty[slot], (use - 1) & 1, &abort_flag, a.err)) break;
           mbar_expect_tx(&bar_full[slot], C::kTileBytes);
-          const CUtensorMap *map = (L & 1) ? &tm_v : &tm_k;
+          const int jg = j0 + (L >> 1);                   // global key tile
+          const bool second = jg >= a.tiles1;
+          const CUtensorMap *map = second ? ((L & 1) ? &tm_v2 : &tm_k2)
+                                          : ((L & 1) ? &tm_v : &tm_k);
+          const int y = (second ? jg - a.tiles1 : jg) * kBN;
           uint8_t *dst = sKV + slot * C::kTileBytes;
 #pragma unroll
           for (int c = 0; c < C::kChunks; ++c)
-            tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64,
-                        (j0 + (L >> 1)) * kBN);
+            tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, y);
           issued = L + 1;
         }
         // Drain: every issued copy has landed before the CTA may exit.
@@ -623,7 +630,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     for (int j = 0; j < nT; ++j) {
       if (!(ok = mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err))) break;
       fence_after();
-      const int valid = a.N - (j0 + j) * kBN;      // keys of this tile that exist
+      const int jg = j0 + j;                       // keys of this tile that exist
+      const int valid = jg < a.tiles1 ? a.rows1 - jg * kBN : a.rows2 - (jg - a.tiles1) * kBN;
       if (valid >= kBN)
         softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
       else
@@ -725,8 +733,10 @@ constexpr int kF32Keys = 32;
 template <int D>
 __global__ void __launch_bounds__(kF32Threads)
 attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
-                const float *__restrict__ kc, const float *__restrict__ vc, float *__restrict__ out,
-                int n_active, int N, int H, int q_rows, float scale, unsigned *err) {
+                const float *__restrict__ kc, const float *__restrict__ vc, int rows1,
+                const float *__restrict__ kb, const float *__restrict__ vb,
+                float *__restrict__ out, int n_active, int N, int H, int q_rows, float scale,
+                unsigned *err) {
   constexpr int TPQ = D / 32;
   constexpr int QPB = kF32Threads / TPQ;
   __shared__ float sK[kF32Keys][D];
@@ -756,10 +766,12 @@ attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
     for (int e = threadIdx.x; e < kF32Keys * D / 4; e += kF32Threads) {
       const int kk = e / (D / 4), d4 = e % (D / 4);
       float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
-      if (n0 + kk < N) {
-        const size_t off = ((size_t)(n0 + kk) * H + h) * D;
-        kv = reinterpret_cast<const float4 *>(kc + off)[d4];
-        vv = reinterpret_cast<const float4 *>(vc + off)[d4];
+      const int key = n0 + kk;
+      if (key < N) {
+        const bool first = key < rows1;
+        const size_t off = ((size_t)(first ? key : key - rows1) * H + h) * D;
+        kv = reinterpret_cast<const float4 *>((first ? kc : kb) + off)[d4];
+        vv = reinterpret_cast<const float4 *>((first ? vc : vb) + off)[d4];
       }
       reinterpret_cast<float4 *>(&sK[kk][0])[d4] = kv;
       reinterpret_cast<float4 *>(&sV[kk][0])[d4] = vv;
@@ -841,8 +853,10 @@ size_t split_workspace_bytes(int D) {
 
 template <int D>
 int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
-              const void *v_cache, int N, int H, float scale, void *out, void *ws,
-              size_t ws_bytes, cudaStream_t stream, unsigned *err) {
+              const void *v_cache, int rows1, const void *k_base, const void *v_base, int rows2,
+              int H, float scale, void *out, void *ws, size_t ws_bytes, cudaStream_t stream,
+              unsigned *err) {
+  const int N = rows1 + rows2;
   using C = TcCfg<D>;
   static std::atomic<int> configured[64];
   int dev = 0;
@@ -859,9 +873,15 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
       return HSA_ERR_CUDA;
     configured[dev].store(1);
   }
-  CUtensorMap mk, mv;
-  if (!make_kv_map(&mk, k_cache, N, H, D) || !make_kv_map(&mv, v_cache, N, H, D))
+  CUtensorMap mk, mv, mk2, mv2;
+  if (rows1 > 0 && (!make_kv_map(&mk, k_cache, rows1, H, D) ||
+                    !make_kv_map(&mv, v_cache, rows1, H, D)))
     return HSA_ERR_CUDA;
+  if (rows2 > 0 && (!make_kv_map(&mk2, k_base, rows2, H, D) ||
+                    !make_kv_map(&mv2, v_base, rows2, H, D)))
+    return HSA_ERR_CUDA;
+  if (rows1 == 0) mk = mk2, mv = mv2;   // unused source: any valid map
+  if (rows2 == 0) mk2 = mk, mv2 = mv;
   TcArgs a;
   a.q = static_cast<const __nv_bfloat16 *>(q);
   a.q_idx = q_idx;
@@ -871,7 +891,10 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.N = N;
   a.H = H;
   a.q_rows = q_idx ? N : n_active;
-  a.n_kv_tiles = (N + kBN - 1) / kBN;
+  a.rows1 = rows1;
+  a.rows2 = rows2;
+  a.tiles1 = (rows1 + kBN - 1) / kBN;
+  a.n_kv_tiles = a.tiles1 + (rows2 + kBN - 1) / kBN;
   a.scale_log2 = scale * 1.4426950408889634f;
   a.inject_stall = g_inject_stall.load(std::memory_order_relaxed);
   // Work plan: one CTA per SM at a time, so U units take ceil(U / sms) waves.
@@ -894,7 +917,7 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.ws_o = pieces > 1 ? static_cast<float *>(ws) : nullptr;
   a.ws_ml = pieces > 1 ? a.ws_o + (size_t)rem * pieces * (kQT * kBM) * D : nullptr;
   const long long grid = (long long)a.n_whole + (pieces > 1 ? (long long)rem * pieces : 0);
-  attn_tc_kernel<D><<<(unsigned)grid, kTcThreads, C::kSmem, stream>>>(mk, mv, a);
+  attn_tc_kernel<D><<<(unsigned)grid, kTcThreads, C::kSmem, stream>>>(mk, mv, mk2, mv2, a);
   if (cudaGetLastError() != cudaSuccess) return HSA_ERR_CUDA;
   if (pieces > 1) {
     const long long warps = (long long)rem * (kQT * kBM);
@@ -906,13 +929,15 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
 
 template <int D>
 int launch_f32(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
-               const void *v_cache, int N, int H, float scale, void *out, cudaStream_t stream,
-               unsigned *err) {
+               const void *v_cache, int rows1, const void *k_base, const void *v_base, int rows2,
+               int H, float scale, void *out, cudaStream_t stream, unsigned *err) {
   constexpr int QPB = kF32Threads / (D / 32);
+  const int N = rows1 + rows2;
   const dim3 grid((n_active + QPB - 1) / QPB, H);
   attn_f32_kernel<D><<<grid, kF32Threads, 0, stream>>>(
       static_cast<const float *>(q), q_idx, static_cast<const float *>(k_cache),
-      static_cast<const float *>(v_cache), static_cast<float *>(out), n_active, N, H,
+      static_cast<const float *>(v_cache), rows1, static_cast<const float *>(k_base),
+      static_cast<const float *>(v_base), static_cast<float *>(out), n_active, N, H,
       q_idx ? N : n_active, scale, err);
   return launch_status();
 }
@@ -928,33 +953,62 @@ extern "C" size_t hsa_active_attention_workspace_bytes(int n_active, int N, int 
   return split_workspace_bytes(D);
 }
 
-extern "C" int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
-                                    const void *k_cache, const void *v_cache, int N, int H,
-                                    int D, float scale, void *out, hsa_dtype dtype,
-                                    void *workspace, size_t workspace_bytes,
-                                    hsa_stream_t stream) {
-  if (n_active < 0 || N < 1 || H < 1) return HSA_ERR_INVALID_ARG;
+namespace {
+
+int attention_two_sources(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
+                          const void *v_cache, int rows1, const void *k_base,
+                          const void *v_base, int rows2, int H, int D, float scale, void *out,
+                          hsa_dtype dtype, void *workspace, size_t workspace_bytes,
+                          hsa_stream_t stream) {
+  const long long N = (long long)rows1 + rows2;
+  if (n_active < 0 || rows1 < 0 || rows2 < 0 || N < 1 || N > 0x7fffffffLL || H < 1)
+    return HSA_ERR_INVALID_ARG;
   if (dtype != HSA_BF16 && dtype != HSA_F32) return HSA_ERR_INVALID_ARG;
   if (D != 64 && D != 128) return HSA_ERR_UNSUPPORTED;
   if ((long long)H * D > (1LL << 24)) return HSA_ERR_UNSUPPORTED;
   if (!q_idx && n_active > N) return HSA_ERR_INVALID_ARG;
   if (n_active == 0) return HSA_OK;
-  if (!q || !k_cache || !v_cache || !out) return HSA_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
+  if (!q || !out || (rows1 > 0 && (!k_cache || !v_cache)) || (rows2 > 0 && (!k_base || !v_base)))
+    return HSA_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out) || (rows1 > 0 && (!aligned16(k_cache) || !aligned16(v_cache))) ||
+      (rows2 > 0 && (!aligned16(k_base) || !aligned16(v_base))))
     return HSA_ERR_INVALID_ARG;
   if (!(scale > 0.f) || !std::isfinite(scale)) scale = 1.f / std::sqrt((float)D);
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   cudaStream_t s = (cudaStream_t)stream;
-  if ((long long)(n_active + kBM * kQT - 1) / (kBM * kQT) > 0x7fffffffLL) return HSA_ERR_UNSUPPORTED;
   if (H > 65535) return HSA_ERR_UNSUPPORTED;
   if (dtype == HSA_BF16)
-    return D == 128 ? launch_tc<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out,
-                                     workspace, workspace_bytes, s, err)
-                    : launch_tc<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out,
-                                    workspace, workspace_bytes, s, err);
-  return D == 128 ? launch_f32<128>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err)
-                  : launch_f32<64>(q, q_idx, n_active, k_cache, v_cache, N, H, scale, out, s, err);
+    return D == 128 ? launch_tc<128>(q, q_idx, n_active, k_cache, v_cache, rows1, k_base, v_base,
+                                     rows2, H, scale, out, workspace, workspace_bytes, s, err)
+                    : launch_tc<64>(q, q_idx, n_active, k_cache, v_cache, rows1, k_base, v_base,
+                                    rows2, H, scale, out, workspace, workspace_bytes, s, err);
+  return D == 128 ? launch_f32<128>(q, q_idx, n_active, k_cache, v_cache, rows1, k_base, v_base,
+                                    rows2, H, scale, out, s, err)
+                  : launch_f32<64>(q, q_idx, n_active, k_cache, v_cache, rows1, k_base, v_base,
+                                   rows2, H, scale, out, s, err);
+}
+
+}  // namespace
+
+extern "C" int hsa_active_attention(const void *q, const int32_t *q_idx, int n_active,
+                                    const void *k_cache, const void *v_cache, int N, int H,
+                                    int D, float scale, void *out, hsa_dtype dtype,
+                                    void *workspace, size_t workspace_bytes,
+                                    hsa_stream_t stream) {
+  if (N < 1) return HSA_ERR_INVALID_ARG;
+  return attention_two_sources(q, q_idx, n_active, k_cache, v_cache, N, nullptr, nullptr, 0, H,
+                               D, scale, out, dtype, workspace, workspace_bytes, stream);
+}
+
+extern "C" int hsa_active_attention_prefix(const void *q, const int32_t *q_idx, int n_active,
+                                           const void *k_cache, const void *v_cache, int M,
+                                           const void *k_base, const void *v_base, int B, int H,
+                                           int D, float scale, void *out, hsa_dtype dtype,
+                                           void *workspace, size_t workspace_bytes,
+                                           hsa_stream_t stream) {
+  return attention_two_sources(q, q_idx, n_active, k_cache, v_cache, M, k_base, v_base, B, H, D,
+                               scale, out, dtype, workspace, workspace_bytes, stream);
 }
 
 extern "C" int hsa_test_inject_attention_stall(int mode) {

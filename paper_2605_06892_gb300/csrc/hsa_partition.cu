@@ -338,6 +338,77 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
   return launch_status();
 }
 
+// ------------------------------------------------------- token reordering
+//
+// Sec. 2.5: new position r holds old token order[r]; non-baseline tokens
+// (group != 0) first, then the baseline group, each in token order.  Same
+// workspace-free scheme as the active set: block b counts the non-baseline
+// tokens before its chunk, then ranks its chunk with warp ballots.
+
+template <bool kVec>
+__global__ void __launch_bounds__(kActThreads)
+reorder_kernel(const int32_t *__restrict__ group_of, int N, int M, int chunk,
+               int32_t *__restrict__ order, int32_t *__restrict__ where,
+               int32_t *__restrict__ group_new, unsigned *err) {
+  __shared__ int warp_cnt[32];
+  __shared__ int block_base;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int start = blockIdx.x * chunk;
+  const int end = min(N, start + chunk);
+  int c = 0;
+  if (kVec) {
+    const int4 *g4 = reinterpret_cast<const int4 *>(group_of);
+    for (int i = threadIdx.x; i < start / 4; i += kActThreads) {
+      const int4 v = __ldg(g4 + i);
+      c += (v.x != 0) + (v.y != 0) + (v.z != 0) + (v.w != 0);
+    }
+  } else {
+    for (int i = threadIdx.x; i < start; i += kActThreads) c += __ldg(group_of + i) != 0;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) warp_cnt[w] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int s = 0;
+    for (int i = 0; i < kActThreads / 32; ++i) s += warp_cnt[i];
+    block_base = s;
+  }
+  __syncthreads();
+  int nb_base = block_base;             // non-baseline tokens before b0
+  for (int b0 = start; b0 < end; b0 += kActThreads) {
+    const int n = b0 + threadIdx.x;
+    int g = 0, flag = 0;
+    if (n < end) {
+      g = group_of[n];
+      flag = g != 0;
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, flag);
+    __syncthreads();
+    if (lane == 0) warp_cnt[w] = __popc(bal);
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int i = 0; i < kActThreads / 32; ++i) {
+      const int v = warp_cnt[i];
+      before += (i < w) ? v : 0;
+      total += v;
+    }
+    if (n < end) {
+      const int nb_rank = nb_base + before + __popc(bal & ((1u << lane) - 1u));
+      // baseline rank = tokens before n that are baseline
+      const int r = flag ? nb_rank : M + (n - nb_rank);
+      if ((flag && nb_rank < M) || (!flag && r < N)) {
+        order[r] = n;
+        if (where) where[n] = r;
+        if (group_new) group_new[r] = g;
+      } else {
+        set_error(err, kErrIndex);
+      }
+    }
+    nb_base += total;
+  }
+}
+
 // ------------------------------------------------- allocation strategies
 //
 // Statistics whose ranking by hsa_partition gives the other token allocation
@@ -425,5 +496,29 @@ extern "C" int hsa_reserve_first_frame(float *stat, int N, int frame_tokens,
   if (!stat) return HSA_ERR_INVALID_ARG;
   const int blocks = (int)std::min<long long>((frame_tokens + 255) / 256, (long long)sm_count() * 8);
   reserve_frame_kernel<<<blocks, 256, 0, (cudaStream_t)stream>>>(stat, frame_tokens);
+  return launch_status();
+}
+
+extern "C" int hsa_reorder_tokens(const int32_t *group_of, int N, int n_baseline,
+                                  int32_t *order, int32_t *where, int32_t *group_new,
+                                  hsa_stream_t stream) {
+  if (N < 0 || n_baseline < 0 || n_baseline > N) return HSA_ERR_INVALID_ARG;
+  if (N == 0) return HSA_OK;
+  if (!group_of || !order) return HSA_ERR_INVALID_ARG;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const int sms = sm_count();
+  long long chunk = ((long long)N + sms - 1) / sms;
+  chunk = ((chunk + kActThreads - 1) / kActThreads) * kActThreads;
+  if (chunk < 4096) chunk = 4096;
+  const int blocks = (int)(((long long)N + chunk - 1) / chunk);
+  const int M = N - n_baseline;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (aligned16(group_of))
+    reorder_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, M, (int)chunk, order, where,
+                                                         group_new, err);
+  else
+    reorder_kernel<false><<<blocks, kActThreads, 0, s>>>(group_of, N, M, (int)chunk, order, where,
+                                                          group_new, err);
   return launch_status();
 }
