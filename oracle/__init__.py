@@ -61,6 +61,8 @@ def lib():
             "orc_uniform_stat": [c_int, c_p],
             "orc_reserve_frame": [c_p, c_int, c_int],
             "orc_reorder": [c_p, c_int, c_p, c_p, c_p],
+            "orc_rope_table": [c_int, c_int, c_int, c_int, c_d, c_p],
+            "orc_rope_rows": [c_p, c_p, c_int, c_int, c_int, c_p, c_int],
         }
         for name, args in sig.items():
             f = getattr(_lib, name)
@@ -236,3 +238,23 @@ def reorder(group_of: torch.Tensor):
     M = _check(lib().orc_reorder(g.data_ptr(), N, order.data_ptr(), where.data_ptr(),
                                  gn.data_ptr()))
     return order[:N].clone(), where[:N].clone(), gn[:N].clone(), M
+
+
+def rope_table(grid, D: int, theta: float = 10000.0) -> torch.Tensor:
+    """fp32 [N, D/2, 2] (cos, sin) table of a (F, Hh, Ww) token grid."""
+    F, Hh, Ww = grid
+    out = torch.empty((F * Hh * Ww, D // 2, 2), dtype=torch.float32)
+    _check(lib().orc_rope_table(F, Hh, Ww, D, float(theta), out.data_ptr()))
+    return out
+
+
+def rope_rows(x: torch.Tensor, idx: torch.Tensor, table: torch.Tensor) -> torch.Tensor:
+    """New bf16 tensor: rows of x [n, H, D] rotated by table[idx[j]]."""
+    assert x.dtype == torch.bfloat16
+    out = x.contiguous().clone()
+    n, H, D = out.shape
+    idx = idx.contiguous().to(torch.int32)
+    table = table.contiguous()
+    _check(lib().orc_rope_rows(out.data_ptr(), idx.data_ptr(), n, H, D, table.data_ptr(),
+                               table.shape[0]))
+    return out

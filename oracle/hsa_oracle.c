@@ -29,6 +29,8 @@
  *   orc_reserve_frame    App. B "first-frame reservation (F)".
  *   orc_reorder          Sec. 2.5 "token reordering": non-baseline tokens
  *                        first, then the baseline group, each in token order.
+ *   orc_rope_table,      Sec. 2.3: rotary position embedding of the active
+ *   orc_rope_rows        rows, their frequencies subsampled (gathered) to A_i.
  *
  * Readings where the paper is silent (each is listed with its reason in the
  * design notes): ties in the ranking go to the lower token index first and
@@ -459,4 +461,79 @@ int orc_reorder(const int32_t *group_of, int N, int32_t *order, int32_t *where,
             ++r;
         }
     return M;
+}
+
+/* ------------------------------------------------------------- rotary (RoPE) */
+
+/* Rotary embedding table of a (F, Hh, Ww) token grid, tokens row-major over
+ * (f, h, w).  Reading (the paper names RoPE but not its layout): the D/2
+ * rotation pairs are split into three bands, p_h = p_w = floor(D/6) pairs for
+ * the row and column axes and p_t = D/2 - 2*p_h for the frame axis, in that
+ * order (t, h, w); pair i of a band with p pairs turns by
+ * pos * theta^(-i/p).  table[n][i] = (cos, sin) of token n's angle for pair
+ * i, computed in fp64 and rounded to fp32 (the table's storage type). */
+int orc_rope_table(int F, int Hh, int Ww, int D, double theta, float *table)
+{
+    if (F < 1 || Hh < 1 || Ww < 1 || D < 2 || (D & 1) || !(theta > 1.0))
+        return ORC_EINVAL;
+    const int P = D / 2, ph = D / 6, pt = P - 2 * (D / 6);
+    for (int f = 0; f < F; ++f)
+        for (int h = 0; h < Hh; ++h)
+            for (int w = 0; w < Ww; ++w) {
+                const size_t n = ((size_t)f * Hh + h) * Ww + w;
+                for (int i = 0; i < P; ++i) {
+                    int band_i, band_p, pos;
+                    if (i < pt) {
+                        band_i = i; band_p = pt; pos = f;
+                    } else if (i < pt + ph) {
+                        band_i = i - pt; band_p = ph; pos = h;
+                    } else {
+                        band_i = i - pt - ph; band_p = ph; pos = w;
+                    }
+                    const double ang = pos * pow(theta, -(double)band_i / band_p);
+                    table[(n * P + i) * 2] = (float)cos(ang);
+                    table[(n * P + i) * 2 + 1] = (float)sin(ang);
+                }
+            }
+    return ORC_OK;
+}
+
+static uint16_t to_bf16(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7fffffffu) > 0x7f800000u)
+        return (uint16_t)((u >> 16) | 0x40u);          /* NaN stays NaN */
+    u += 0x7fffu + ((u >> 16) & 1u);                    /* round to nearest even */
+    return (uint16_t)(u >> 16);
+}
+
+/* Rotate rows j < n of a bf16 tensor x[n][H][D] in place by the table row of
+ * their token idx[j] (the frequencies subsampled to the active set):
+ * (x0, x1) -> (x0 c - x1 s, x0 s + x1 c) per pair, as
+ * y0 = fma(x0, c, -(x1 s)), y1 = fma(x0, s, x1 c) in fp32, rounded to bf16. */
+int orc_rope_rows(uint16_t *x, const int32_t *idx, int n, int H, int D, const float *table,
+                  int N)
+{
+    const int P = D / 2;
+    for (int j = 0; j < n; ++j) {
+        if (idx[j] < 0 || idx[j] >= N)
+            return ORC_EINDEX;
+        const float *t = table + (size_t)idx[j] * P * 2;
+        for (int h = 0; h < H; ++h) {
+            uint16_t *row = x + ((size_t)j * H + h) * D;
+            for (int i = 0; i < P; ++i) {
+                uint32_t a = (uint32_t)row[2 * i] << 16, b = (uint32_t)row[2 * i + 1] << 16;
+                float x0, x1;
+                memcpy(&x0, &a, 4);
+                memcpy(&x1, &b, 4);
+                const float c = t[2 * i], s = t[2 * i + 1];
+                const float y0 = fmaf(x0, c, -(x1 * s));
+                const float y1 = fmaf(x0, s, x1 * c);
+                row[2 * i] = to_bf16(y0);
+                row[2 * i + 1] = to_bf16(y1);
+            }
+        }
+    }
+    return ORC_OK;
 }

@@ -562,3 +562,42 @@ def test_reordered_cache_gives_the_same_attention():
         assert torch.equal(torch.sort(old_of_new).values.to(torch.int32), idx)
         perm = torch.argsort(old_of_new)
         assert torch.allclose(got[perm], ref, atol=1e-12)
+
+
+# ------------------------------------------------------------------- RoPE
+
+def test_rope_table_bands_and_standard_frequencies():
+    """Each band is standard RoPE along its axis: the first pair of every band
+    turns by the axis position in radians, pair i by pos * theta^(-i/p); a
+    token at the origin is not rotated."""
+    grid, D = (3, 4, 5), 128
+    tab = oracle.rope_table(grid, D).double()
+    P, ph = D // 2, D // 6
+    pt = P - 2 * ph
+    assert (pt, ph) == (22, 21)
+    assert torch.all(tab[0, :, 0] == 1.0) and torch.all(tab[0, :, 1] == 0.0)
+    n = (2 * 4 + 3) * 5 + 1                     # f = 2, h = 3, w = 1
+    for i, pos, p, bi in ((0, 2, pt, 0), (pt, 3, ph, 0), (pt + ph, 1, ph, 0),
+                          (5, 2, pt, 5), (pt + 7, 3, ph, 7), (P - 1, 1, ph, ph - 1)):
+        ang = pos * 10000.0 ** (-bi / p)
+        assert abs(tab[n, i, 0] - math.cos(ang)) < 1e-7
+        assert abs(tab[n, i, 1] - math.sin(ang)) < 1e-7
+
+
+def test_rope_rotation_invariants():
+    """Rotation keeps each pair's norm, and the dot product of two rotated
+    vectors depends only on their position difference (relative encoding)."""
+    grid, D = (4, 4, 4), 64
+    tab = oracle.rope_table(grid, D)
+    x = synth.normal((2, 1, D), 3, "bf16")
+    pos = lambda f, h, w: (f * 4 + h) * 4 + w  # noqa: E731
+    rot = lambda v, n: oracle.rope_rows(v, torch.tensor([n], dtype=torch.int32), tab)  # noqa: E731
+    a, b = x[:1], x[1:]
+    ra = rot(a, pos(1, 2, 0)).double()
+    assert torch.allclose(ra.view(-1, 2).norm(dim=1), a.double().view(-1, 2).norm(dim=1),
+                          rtol=1e-2)
+    d1 = (rot(a, pos(1, 2, 0)).double() * rot(b, pos(2, 3, 1)).double()).sum()
+    d2 = (rot(a, pos(2, 0, 2)).double() * rot(b, pos(3, 1, 3)).double()).sum()
+    assert abs(float(d1 - d2)) < 0.15
+    # the identity row leaves the vector unchanged
+    assert torch.equal(rot(a, 0), a)
