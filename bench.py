@@ -531,6 +531,12 @@ def memory_sweep():
         vf = torch.empty_like(kf).normal_()
         ms = timed(lambda: hsa.hsa_kv_sync_scatter(kc, vc, kf, vf, idx, n, stream))
         report("kv_scatter", f"{n} rows x 2 x {row} B", n * (4 * row + 4), ms)
+        if n in (32768, 262144):
+            tab = torch.empty((N, 64, 2), device=dev).uniform_(-1, 1)
+            ms = timed(lambda: hsa.hsa_kv_sync_scatter_rope(kc, vc, kf, vf, idx, n, tab, stream))
+            # K, V read and written, idx, and the token's 512-byte table row
+            report("kv_scatter_rope", f"{n} rows x 2 x {row} B", n * (4 * row + 4 + 512), ms)
+            del tab
         del kc, vc, kf, vf
     for C in (16, 128):
         for N in (1 << 16, 1 << 20, 1 << 22, 1 << 24):

@@ -218,6 +218,31 @@ int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_fresh,
                         int N, int H, int D, hsa_dtype dtype,
                         hsa_stream_t stream);
 
+/* Rotary position embedding of the active rows (Sec. 2.3: the positional
+ * frequencies are subsampled to match A_i).  The table holds, for every token
+ * n of the grid and rotation pair i, (cos, sin) of its angle; the calls below
+ * rotate an active row j by the table row of its token idx[j], pair (x0, x1)
+ * of each head becoming (fma(x0, c, -(x1 s)), fma(x0, s, x1 c)) in fp32,
+ * rounded to bf16.
+ *
+ * hsa_rope_table: host-side table of a (F, Hh, Ww) grid, tokens row-major:
+ * the D/2 pairs form three bands, p_t = D/2 - 2 floor(D/6) pairs for the
+ * frame, then floor(D/6) each for the row and the column; pair i of a band
+ * of p pairs turns by pos * theta^(-i/p).  table: host, fp32 [N, D/2, 2]
+ * written (fp64 math, rounded once).  D a multiple of 8.
+ *
+ * hsa_rope_rows: x device bf16 [n, H, D], rotated in place (e.g. Q[A_i]).
+ * hsa_kv_sync_scatter_rope: hsa_kv_sync_scatter (bf16) with the fresh K rows
+ * rotated on their way into the cache; V is copied unchanged.
+ *   table  device, fp32 [N, D/2, 2], 16-byte aligned.
+ * An idx entry outside [0, N) skips its row (HSA_ERR_INDEX). */
+int hsa_rope_table(int F, int Hh, int Ww, int D, double theta, float *table);
+int hsa_rope_rows(void *x, const int32_t *idx, int n, int H, int D, const float *table, int N,
+                  hsa_stream_t stream);
+int hsa_kv_sync_scatter_rope(void *k_cache, void *v_cache, const void *k_fresh,
+                             const void *v_fresh, const int32_t *idx, int n_active, int N,
+                             int H, int D, const float *table, hsa_stream_t stream);
+
 /* -------------------------------------------------- a5 active attention */
 
 /* Full-context attention of the active queries (Sec. 2.3, step 3; Sec. 2.1

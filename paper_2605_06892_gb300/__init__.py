@@ -22,7 +22,8 @@ __all__ = [
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
     "hsa_partition", "hsa_partition_static", "hsa_uniform_stat", "hsa_reserve_first_frame",
     "hsa_reorder_tokens", "hsa_partition_active", "hsa_gather_active",
-    "hsa_kv_sync_scatter", "hsa_active_attention", "hsa_active_attention_prefix",
+    "hsa_kv_sync_scatter", "hsa_rope_table", "hsa_rope_rows", "hsa_kv_sync_scatter_rope",
+    "hsa_active_attention", "hsa_active_attention_prefix",
     "hsa_active_attention_workspace_bytes",
     "hsa_cached_euler", "hsa_cached_euler_l1rel",
     "hsa_get_device_error", "hsa_test_inject_attention_stall",
@@ -70,6 +71,10 @@ _SIGS = {
     "hsa_active_attention_prefix": ([_c_p, _c_p, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p, _c_int,
                                      _c_int, _c_int, _c_f, _c_p, _c_int, _c_p, _c_sz, _c_p],
                                     _c_int),
+    "hsa_rope_table": ([_c_int, _c_int, _c_int, _c_int, _c_d, _c_p], _c_int),
+    "hsa_rope_rows": ([_c_p, _c_p, _c_int, _c_int, _c_int, _c_p, _c_int, _c_p], _c_int),
+    "hsa_kv_sync_scatter_rope": ([_c_p, _c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_int,
+                                  _c_p, _c_p], _c_int),
     "hsa_reorder_tokens": ([_c_p, _c_int, _c_int, _c_p, _c_p, _c_p, _c_p], _c_int),
     "hsa_active_attention_workspace_bytes": ([_c_int, _c_int, _c_int, _c_int, _c_int], _c_sz),
     "hsa_cached_euler": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p], _c_int),
@@ -224,6 +229,28 @@ def hsa_kv_sync_scatter(k_cache, v_cache, k_fresh, v_fresh, idx, n_active: int,
     _check(lib().hsa_kv_sync_scatter(_p(k_cache), _p(v_cache), _p(k_fresh), _p(v_fresh),
                                      _p(idx), n_active, N, H, D, _dtype_code(k_cache),
                                      _stream(stream)), "hsa_kv_sync_scatter")
+
+
+def hsa_rope_table(grid, D: int, theta: float = 10000.0) -> torch.Tensor:
+    """Host fp32 [N, D/2, 2] (cos, sin) table of a (F, Hh, Ww) token grid."""
+    F, Hh, Ww = grid
+    out = torch.empty((F * Hh * Ww, D // 2, 2), dtype=torch.float32)
+    _check(lib().hsa_rope_table(F, Hh, Ww, D, float(theta), out.data_ptr()), "hsa_rope_table")
+    return out
+
+
+def hsa_rope_rows(x, idx, n: int, table, stream=None) -> None:
+    _, H, D = x.shape
+    _check(lib().hsa_rope_rows(_p(x), _p(idx), n, H, D, _p(table), table.shape[0],
+                               _stream(stream)), "hsa_rope_rows")
+
+
+def hsa_kv_sync_scatter_rope(k_cache, v_cache, k_fresh, v_fresh, idx, n_active: int, table,
+                             stream=None) -> None:
+    N, H, D = k_cache.shape
+    _check(lib().hsa_kv_sync_scatter_rope(_p(k_cache), _p(v_cache), _p(k_fresh), _p(v_fresh),
+                                          _p(idx), n_active, N, H, D, _p(table),
+                                          _stream(stream)), "hsa_kv_sync_scatter_rope")
 
 
 def hsa_active_attention_prefix(q, q_idx, n_active: int, k_cache, v_cache, k_base, v_base, out,

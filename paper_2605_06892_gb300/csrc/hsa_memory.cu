@@ -8,6 +8,10 @@
 // or store.  Each lane keeps several vectors in flight before storing.
 // The row index is read once per row by its lane group; indices are checked
 // against the row count and a bad one skips its row and sets the error word.
+#include <cuda_bf16.h>
+
+#include <cmath>
+
 #include "hsa_internal.cuh"
 
 namespace hsa {
@@ -239,6 +243,96 @@ euler_l1rel_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
   }
 }
 
+// Rotary position embedding of the active rows (Sec. 2.3: the positional
+// frequencies are subsampled to A_i): row j of a token tensor is rotated by
+// the (cos, sin) table row of its token idx[j].  One 16-byte vector holds 8
+// bf16 values = 4 rotation pairs; pair (x0, x1) becomes
+// (fma(x0, c, -(x1 s)), fma(x0, s, x1 c)) in fp32, rounded to bf16.
+__device__ __forceinline__ uint4 rope8(uint4 v, const float4 *tab) {
+  uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float4 cs2 = __ldg(tab + (k >> 1));          // (c, s) of two pairs
+    const float c = (k & 1) ? cs2.z : cs2.x, s = (k & 1) ? cs2.w : cs2.y;
+    const float x0 = __uint_as_float(w[k] << 16), x1 = __uint_as_float(w[k] & 0xffff0000u);
+    const float y0 = __fmaf_rn(x0, c, -(x1 * s));
+    const float y1 = __fmaf_rn(x0, s, x1 * c);
+    const __nv_bfloat162 r = __floats2bfloat162_rn(y0, y1);
+    w[k] = *reinterpret_cast<const uint32_t *>(&r);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// In-place rotation of rows j < n of x [n, H*D] (bf16): a lane group owns a
+// row; vector c covers head 8c / D and pairs ((8c) % D)/2 .. +3.
+__global__ void __launch_bounds__(kThreads)
+rope_rows_kernel(uint4 *__restrict__ x, const int32_t *__restrict__ idx, int n, int vecs, int D,
+                 const float4 *__restrict__ table, int N, int lpr_log2, unsigned *err) {
+  const int L = 1 << lpr_log2;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> lpr_log2, sl = lane & (L - 1);
+  const int rows_per_warp = 32 >> lpr_log2;
+  const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+  const int pairs = D / 2;
+  for (long long j = warp * rows_per_warp + sub; j < n; j += nwarps * rows_per_warp) {
+    const int t = __ldg(idx + j);
+    if (t < 0 || t >= N) {
+      set_error(err, kErrIndex);
+      continue;
+    }
+    const float4 *trow = table + (size_t)t * (pairs / 2);
+    uint4 *row = x + j * vecs;
+    for (int v = sl; v < vecs; v += L) {
+      const int pair0 = ((v * 8) % D) / 2;
+      row[v] = rope8(row[v], trow + pair0 / 2);
+    }
+  }
+}
+
+// KV-cache synchronisation with K rotated on the way in: rows 0..n-1 are K
+// rows (rotated by the table row of token idx[j]), rows n..2n-1 the V rows
+// (copied).
+__global__ void __launch_bounds__(kThreads)
+kv_scatter_rope_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
+                       const uint4 *__restrict__ kf, const uint4 *__restrict__ vf,
+                       const int32_t *__restrict__ idx, int n_active, int N, int vecs, int D,
+                       const float4 *__restrict__ table, int lpr_log2, unsigned *err) {
+  const int L = 1 << lpr_log2;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> lpr_log2, sl = lane & (L - 1);
+  const int rows_per_warp = 32 >> lpr_log2;
+  const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+  const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+  const int pairs = D / 2;
+  for (long long jj = warp * rows_per_warp + sub; jj < 2LL * n_active;
+       jj += nwarps * rows_per_warp) {
+    const bool is_v = jj >= n_active;
+    const long long j = is_v ? jj - n_active : jj;
+    const int r = __ldg(idx + j);
+    if (r < 0 || r >= N) {
+      if (!is_v) set_error(err, kErrIndex);
+      continue;
+    }
+    const uint4 *s = (is_v ? vf : kf) + j * vecs;
+    uint4 *d = (is_v ? vc : kc) + (long long)r * vecs;
+    const float4 *trow = table + (size_t)r * (pairs / 2);
+    for (int v0 = sl; v0 < vecs; v0 += kScatterUnroll * L) {
+      uint4 buf[kScatterUnroll];
+#pragma unroll
+      for (int u = 0; u < kScatterUnroll; ++u) {
+        const int v = v0 + u * L;
+        if (v < vecs) buf[u] = ld_stream(s + v);
+      }
+#pragma unroll
+      for (int u = 0; u < kScatterUnroll; ++u) {
+        const int v = v0 + u * L;
+        if (v < vecs) d[v] = is_v ? buf[u] : rope8(buf[u], trow + (((v * 8) % D) / 2) / 2);
+      }
+    }
+  }
+}
+
 // Grid for n_rows rows handled by lane groups of size L: up to 8 blocks of
 // 256 threads per SM (a full SM), no more than the rows need; blocks beyond
 // what is resident wait their turn.
@@ -348,5 +442,62 @@ extern "C" int hsa_cached_euler_l1rel(float *x, float *v_cache, const float *v_f
                        (cudaStream_t)stream>>>(
       (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, N, vecs, log2i(L), dsigma,
       n_fresh, stat, weight, err);
+  return launch_status();
+}
+
+extern "C" int hsa_rope_table(int F, int Hh, int Ww, int D, double theta, float *table) {
+  if (F < 1 || Hh < 1 || Ww < 1 || D < 8 || (D & 7) || !(theta > 1.0) || !table)
+    return HSA_ERR_INVALID_ARG;
+  const int P = D / 2, ph = D / 6, pt = P - 2 * ph;
+  for (int f = 0; f < F; ++f)
+    for (int h = 0; h < Hh; ++h)
+      for (int w = 0; w < Ww; ++w) {
+        const size_t n = ((size_t)f * Hh + h) * Ww + w;
+        for (int i = 0; i < P; ++i) {
+          const bool tb = i < pt, hb = !tb && i < pt + ph;
+          const int bi = tb ? i : (hb ? i - pt : i - pt - ph);
+          const int bp = tb ? pt : ph;
+          const int pos = tb ? f : (hb ? h : w);
+          const double ang = (double)pos * std::pow(theta, -(double)bi / (double)bp);
+          table[(n * P + i) * 2] = (float)std::cos(ang);
+          table[(n * P + i) * 2 + 1] = (float)std::sin(ang);
+        }
+      }
+  return HSA_OK;
+}
+
+extern "C" int hsa_rope_rows(void *x, const int32_t *idx, int n, int H, int D,
+                             const float *table, int N, hsa_stream_t stream) {
+  if (n < 0 || H < 1 || D < 8 || (D & 7) || N < 1) return HSA_ERR_INVALID_ARG;
+  if (n == 0) return HSA_OK;
+  if (!x || !idx || !table || !aligned16(x) || !aligned16(table)) return HSA_ERR_INVALID_ARG;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const long long vecs = (long long)H * D / 8;
+  if (vecs > (1LL << 30)) return HSA_ERR_UNSUPPORTED;
+  const int L = lanes_per_row(vecs);
+  rope_rows_kernel<<<grid_for(n, L), kThreads, 0, (cudaStream_t)stream>>>(
+      (uint4 *)x, idx, n, (int)vecs, D, (const float4 *)table, N, log2i(L), err);
+  return launch_status();
+}
+
+extern "C" int hsa_kv_sync_scatter_rope(void *k_cache, void *v_cache, const void *k_fresh,
+                                        const void *v_fresh, const int32_t *idx, int n_active,
+                                        int N, int H, int D, const float *table,
+                                        hsa_stream_t stream) {
+  if (N < 0 || n_active < 0 || H < 1 || D < 8 || (D & 7)) return HSA_ERR_INVALID_ARG;
+  if (n_active == 0) return HSA_OK;
+  if (!k_cache || !v_cache || !k_fresh || !v_fresh || !idx || !table) return HSA_ERR_INVALID_ARG;
+  if (!aligned16(k_cache) || !aligned16(v_cache) || !aligned16(k_fresh) || !aligned16(v_fresh) ||
+      !aligned16(table))
+    return HSA_ERR_INVALID_ARG;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const long long vecs = (long long)H * D / 8;
+  if (vecs > (1LL << 30)) return HSA_ERR_UNSUPPORTED;
+  const int L = lanes_per_row(vecs);
+  kv_scatter_rope_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
+      (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
+      n_active, N, (int)vecs, D, (const float4 *)table, log2i(L), err);
   return launch_status();
 }

@@ -6,6 +6,7 @@ import os
 import re
 
 import pytest
+import torch
 
 import oracle
 import synth
@@ -87,3 +88,10 @@ def test_workspace_size_is_monotone(hsa):
     sizes = [hsa.hsa_partition_workspace_bytes(n) for n in (1, 4096, 4097, 75600, 10 ** 6)]
     assert sizes == sorted(sizes) and sizes[0] > 0
     assert all(s % 256 == 0 for s in sizes)
+
+
+def test_rope_table_matches_oracle(hsa):
+    for grid, D in (((3, 4, 5), 128), ((2, 3, 3), 64), ((1, 1, 7), 8)):
+        a = hsa.hsa_rope_table(grid, D)
+        b = oracle.rope_table(grid, D)
+        assert torch.allclose(a, b, rtol=0, atol=1e-7)
