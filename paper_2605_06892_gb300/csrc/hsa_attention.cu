@@ -345,26 +345,32 @@ __host__ __device__ inline CtaWork cta_work(int b, int n_qblocks, int n_whole, i
 template <int D, bool kTail>
 __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid, bool first,
                                              float sl2, float &m_run, float &l_run) {
+  // The second half of S is read while the first half's maximum is formed.
   uint32_t r[128];
   tmem_ld32(tS, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
   tmem_ld32(tS + 32, *reinterpret_cast<uint32_t(*)[32]>(&r[32]));
+  tmem_wait_ld();
   tmem_ld32(tS + 64, *reinterpret_cast<uint32_t(*)[32]>(&r[64]));
   tmem_ld32(tS + 96, *reinterpret_cast<uint32_t(*)[32]>(&r[96]));
-  tmem_wait_ld();
-  if (kTail) {
-#pragma unroll
-    for (int i = 0; i < 128; ++i)
-      if (i >= valid) r[i] = __float_as_uint(-INFINITY);
-  }
+  // pm[p] = maximum of scores 16p .. 16p+15: seven three-input steps cover
+  // 16p+1 .. 16p+14, the last step adds 16p+15.
   float pm[8];
 #pragma unroll
-  for (int p = 0; p < 8; ++p) {
-    float m = __uint_as_float(r[16 * p]);
+  for (int half = 0; half < 2; ++half) {
+    if (half == 1) tmem_wait_ld();
+    if (kTail) {
 #pragma unroll
-    for (int i = 1; i < 16; i += 2)
-      m = max3f(m, __uint_as_float(r[16 * p + i]), __uint_as_float(r[16 * p + i + 1]));
-    m = fmaxf(m, __uint_as_float(r[16 * p + 15]));
-    pm[p] = m;
+      for (int i = 64 * half; i < 64 * half + 64; ++i)
+        if (i >= valid) r[i] = __float_as_uint(-INFINITY);
+    }
+#pragma unroll
+    for (int p = 4 * half; p < 4 * half + 4; ++p) {
+      float m = __uint_as_float(r[16 * p]);
+#pragma unroll
+      for (int i = 1; i < 15; i += 2)
+        m = max3f(m, __uint_as_float(r[16 * p + i]), __uint_as_float(r[16 * p + i + 1]));
+      pm[p] = fmaxf(m, __uint_as_float(r[16 * p + 15]));
+    }
   }
   const float mx = fmaxf(max3f(pm[0], pm[1], pm[2]),
                          fmaxf(max3f(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])));
