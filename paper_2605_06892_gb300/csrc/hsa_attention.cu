@@ -18,10 +18,11 @@
 //               the S columns, and at the end normalises O and stores it.
 //   all warps   load the 256 query rows once, by index, into swizzled smem.
 // The two Q tiles ping-pong: while one softmax group works on its scores the
-// tensor core runs the other tile's MMAs.  The running maximum is only moved
-// (and O rescaled in TMEM) when it grows by more than 2^8, so most iterations
-// skip the rescale; the final division by the running sum makes the result
-// exact whatever maximum was used.
+// tensor core runs the other tile's MMAs.  After the first key tile the
+// probabilities are formed against the running reference maximum without
+// computing the tile's maximum; only if a row sum would pass 2^32 is the tile
+// redone with its exact maximum (and O rescaled in TMEM).  The final division
+// by the running sum makes the result exact whatever reference was used.
 // Registers: the block launches at 168 per thread; the first warpgroup then
 // gives registers back (setmaxnreg.dec to 88) and the two softmax warpgroups
 // take them (setmaxnreg.inc to 208): 128*88 + 256*208 = 384*168.
@@ -280,7 +281,6 @@ constexpr int kRegsHigh = 208;           // softmax warpgroups
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kTcThreads * kLaunchRegs,
               "register split exceeds the launch allocation");
 constexpr int kTmemCols = 512;
-constexpr float kRescaleLog2 = 8.0f;   // lazy rescale threshold, log2 units
 
 template <int D>
 struct TcCfg {
@@ -336,59 +336,15 @@ __host__ __device__ inline CtaWork cta_work(int b, int n_qblocks, int n_whole, i
   return w;
 }
 
-// Scores of one 128-key tile for this thread's row: S from TMEM (one read),
-// the running maximum (moved only when it grows by more than 2^8, with O
-// rescaled in TMEM), P = 2^(s*scale*log2e - m) as bf16 pairs written over the
-// first 64 S columns, and the running sum.  kTail masks keys >= valid (the
-// last, ragged tile); full tiles take no per-key test.  Reductions use eight
-// independent partial results to keep dependency chains short.
-template <int D, bool kTail>
-__device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid, bool first,
-                                             float sl2, float &m_run, float &l_run) {
-  // The second half of S is read while the first half's maximum is formed.
-  uint32_t r[128];
-  tmem_ld32(tS, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
-  tmem_ld32(tS + 32, *reinterpret_cast<uint32_t(*)[32]>(&r[32]));
-  tmem_wait_ld();
-  tmem_ld32(tS + 64, *reinterpret_cast<uint32_t(*)[32]>(&r[64]));
-  tmem_ld32(tS + 96, *reinterpret_cast<uint32_t(*)[32]>(&r[96]));
-  // pm[p] = maximum of scores 16p .. 16p+15: seven three-input steps cover
-  // 16p+1 .. 16p+14, the last step adds 16p+15.
-  float pm[8];
-#pragma unroll
-  for (int half = 0; half < 2; ++half) {
-    if (half == 1) tmem_wait_ld();
-    if (kTail) {
-#pragma unroll
-      for (int i = 64 * half; i < 64 * half + 64; ++i)
-        if (i >= valid) r[i] = __float_as_uint(-INFINITY);
-    }
-#pragma unroll
-    for (int p = 4 * half; p < 4 * half + 4; ++p) {
-      float m = __uint_as_float(r[16 * p]);
-#pragma unroll
-      for (int i = 1; i < 15; i += 2)
-        m = max3f(m, __uint_as_float(r[16 * p + i]), __uint_as_float(r[16 * p + i + 1]));
-      pm[p] = fmaxf(m, __uint_as_float(r[16 * p + 15]));
-    }
-  }
-  const float mx = fmaxf(max3f(pm[0], pm[1], pm[2]),
-                         fmaxf(max3f(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-  const float m_new = fmaxf(m_run, mx * sl2);
-  // The reference maximum moves only on the first tile or when it grows by
-  // more than 2^kRescaleLog2; then O (in TMEM) and the sum take the factor
-  // alpha.  O is rescaled after P is written, when the scores are dead.
-  const bool need = first || m_new > m_run + kRescaleLog2;
-  const float alpha = (need && !first) ? fast_exp2(m_run - m_new) : 1.f;
-  if (need) {
-    l_run *= alpha;
-    m_run = m_new;
-  }
+// P = 2^(s*scale*log2e - m) for this thread's 128 scores, as bf16 pairs
+// written over the first 64 S columns (all scores are in registers, so P may
+// overwrite S); returns the row sum of the fp32 values.
+__device__ __forceinline__ float exp_store_tile(uint32_t tS, const uint32_t (&r)[128],
+                                                float sl2, float m) {
   // x = s*scale*log2e - m for a pair of scores in one packed FMA; p = 2^x.
   const uint64_t scale2 = pack2(__float_as_uint(sl2), __float_as_uint(sl2));
-  const uint64_t negm2 = pack2(__float_as_uint(-m_run), __float_as_uint(-m_run));
+  const uint64_t negm2 = pack2(__float_as_uint(-m), __float_as_uint(-m));
   uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
-  // All 128 scores are in registers, so P may overwrite S column by column.
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     uint32_t pk[32];
@@ -404,18 +360,79 @@ __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid
   }
   const uint64_t s01 = add2(ps[0], ps[1]), s23 = add2(ps[2], ps[3]);
   const uint64_t st = add2(s01, s23);
-  l_run += lo_f(st) + hi_f(st);
+  return lo_f(st) + hi_f(st);
+}
+
+// One 128-key tile of this thread's row.  softmax(s) V = sum 2^(c s - m) v /
+// sum 2^(c s - m) holds for any reference m as long as nothing overflows, and
+// m_run (a maximum of earlier tiles) never exceeds the row's true maximum, so
+// after the first tile P is formed against m_run without looking at this
+// tile's maximum (fast path).  If a row's sum then exceeds 2^32 (or is not
+// finite) the warp redoes the tile on the exact path: the row maximum of the
+// scores (still in registers) becomes the new reference, O (in TMEM, idle
+// now: this tile's S is complete, so the previous O += P V is too) and the
+// running sum take the factor 2^(m_old - m_new), and P is formed again.  The
+// first tile always takes the exact path.  kTail masks keys >= valid (the
+// last, ragged tile); full tiles take no per-key test.
+template <int D, bool kTail>
+__device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid, bool first,
+                                             float sl2, float &m_run, float &l_run) {
+  // The second half of S is read while the first half is masked.
+  uint32_t r[128];
+  tmem_ld32(tS, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
+  tmem_ld32(tS + 32, *reinterpret_cast<uint32_t(*)[32]>(&r[32]));
+  tmem_wait_ld();
+  tmem_ld32(tS + 64, *reinterpret_cast<uint32_t(*)[32]>(&r[64]));
+  tmem_ld32(tS + 96, *reinterpret_cast<uint32_t(*)[32]>(&r[96]));
+  if (kTail) {
+#pragma unroll
+    for (int i = 0; i < 64; ++i)
+      if (i >= valid) r[i] = __float_as_uint(-INFINITY);
+  }
+  tmem_wait_ld();
+  if (kTail) {
+#pragma unroll
+    for (int i = 64; i < 128; ++i)
+      if (i >= valid) r[i] = __float_as_uint(-INFINITY);
+  }
+  if (!first) {
+    const float rs = exp_store_tile(tS, r, sl2, m_run);
+    const bool bad = !(rs <= 4294967296.0f);
+    if (!__any_sync(0xffffffffu, bad)) {
+      l_run += rs;
+      return;
+    }
+    tmem_wait_st();   // the exact path rewrites the same P columns
+  }
+  // Exact path.  pm[p] = maximum of scores 16p .. 16p+15: seven
+  // three-input steps cover 16p+1 .. 16p+14, the last step adds 16p+15.
+  float pm[8];
+#pragma unroll
+  for (int p = 0; p < 8; ++p) {
+    float m = __uint_as_float(r[16 * p]);
+#pragma unroll
+    for (int i = 1; i < 15; i += 2)
+      m = max3f(m, __uint_as_float(r[16 * p + i]), __uint_as_float(r[16 * p + i + 1]));
+    pm[p] = fmaxf(m, __uint_as_float(r[16 * p + 15]));
+  }
+  const float mx = fmaxf(max3f(pm[0], pm[1], pm[2]),
+                         fmaxf(max3f(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+  const float m_new = fmaxf(m_run, mx * sl2);
+  const float alpha = (!first && m_new > m_run) ? fast_exp2(m_run - m_new) : 1.f;
+  l_run = first ? 0.f : l_run * alpha;
+  m_run = m_new;
   if (!first && __any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll
-    for (int c = 0; c < D / 32; ++c) {
-      uint32_t o[32];
-      tmem_ld32(tO + 32 * c, o);
+    for (int c = 0; c < D / 16; ++c) {
+      uint32_t o[16];
+      tmem_ld16(tO + 16 * c, o);
       tmem_wait_ld();
 #pragma unroll
-      for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-      tmem_st32(tO + 32 * c, o);
+      for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+      tmem_st16(tO + 16 * c, o);
     }
   }
+  l_run += exp_store_tile(tS, r, sl2, m_run);
 }
 
 template <int D>

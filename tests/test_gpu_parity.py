@@ -338,6 +338,23 @@ def test_attention_large_scores_rescale(hsa):
     _check_attention(out, oracle.attention(q, kc, vc, q_idx=idx), "bf16")
 
 
+@pytest.mark.parametrize("trend", ["growing", "shrinking"])
+def test_attention_score_trends(hsa, trend):
+    """Key norms that grow (or shrink) along the sequence: with growing keys
+    later tiles exceed the first tile's reference maximum by a wide margin
+    (large probabilities, and the exact path once a row sum passes 2^32);
+    with shrinking keys the first tile's reference dominates."""
+    N, H, D, n = 3000, 2, 128, 500
+    ramp = torch.linspace(0.2, 3.0, N) if trend == "growing" else torch.linspace(3.0, 0.2, N)
+    q = synth.normal((n, H, D), 71, "bf16")
+    kc = (synth.normal((N, H, D), 72) * ramp.view(N, 1, 1)).to(torch.bfloat16)
+    vc = synth.normal((N, H, D), 73, "bf16")
+    out = torch.empty((n, H, D), dtype=torch.bfloat16, device=DEV)
+    hsa.hsa_active_attention(q.to(DEV), None, n, kc.to(DEV), vc.to(DEV), out)
+    _no_device_error(hsa)
+    _check_attention(out, oracle.attention(q, kc, vc), "bf16")
+
+
 def _sampled_rows(n_act, k, seed):
     """k random rows plus rows of the last Q block: its first 4 and last 12
     (its tail is ragged whenever n_act is not a multiple of 256)."""
