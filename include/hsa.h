@@ -258,7 +258,7 @@ int hsa_kv_sync_scatter_rope(void *k_cache, void *v_cache, const void *k_fresh,
  *                     hsa_active_attention_workspace_bytes.  With it, the
  *                     (query block, head) units of the last, partly filled
  *                     wave of CTAs are split along the keys and merged
- *                     afterwards, so that wave runs as full as the others;
+ *                     afterwards, so that the last wave finishes sooner;
  *                     without it the result is the same up to rounding order.
  *                     Overwritten; calls using one workspace must not overlap.
  * Supported: D in {64, 128}; H >= 1; 1 <= N < 2^31; 0 <= n_active.

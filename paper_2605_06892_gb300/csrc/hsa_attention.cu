@@ -35,6 +35,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 
@@ -868,10 +869,29 @@ bool make_kv_map(CUtensorMap *map, const void *base, int N, int H, int D) {
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Bytes of split-unit workspace for head dimension D: at most one piece per
+// Bytes of split-unit workspace for head dimension D: at most two pieces per
 // SM, kQT*kBM rows each, D fp32 of O plus (m, l).
 size_t split_workspace_bytes(int D) {
-  return (size_t)sm_count() * (kQT * kBM) * ((size_t)D * 4 + 8) + 512;
+  return 2 * (size_t)sm_count() * (kQT * kBM) * ((size_t)D * 4 + 8) + 512;
+}
+
+// Pieces per tail unit.  The rem units of the last wave, cut into P key
+// ranges each, occupy ceil(rem*P / sms) waves of 1/P unit: minimise that,
+// plus 0.005 unit per piece for its extra prologue, partial write and merge,
+// with at most two waves of pieces and at least one key tile per piece.
+int tail_pieces(int rem, int sms, int n_kv_tiles) {
+  if (rem <= 0) return 1;
+  int best = 1;
+  double best_cost = 1.0 + 0.005;
+  const int pmax = std::min(n_kv_tiles, (2 * sms) / rem);
+  for (int p = 2; p <= pmax; ++p) {
+    const double cost = (double)((rem * p + sms - 1) / sms) / p + 0.005 * p;
+    if (cost < best_cost - 1e-12) {
+      best_cost = cost;
+      best = p;
+    }
+  }
+  return best;
 }
 
 template <int D>
@@ -922,7 +942,8 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.inject_stall = g_inject_stall.load(std::memory_order_relaxed);
   // Work plan: one CTA per SM at a time, so U units take ceil(U / sms) waves.
   // With a workspace, the rem = U mod sms units of the last wave are split
-  // along the keys into `pieces` ranges that fill that wave, then combined.
+  // along the keys into `pieces` ranges (tail_pieces) that shorten that wave,
+  // then combined.
   a.n_qblocks = (n_active + kQT * kBM - 1) / (kQT * kBM);
   const long long units = (long long)a.n_qblocks * H;
   if (units > 0x7fffffffLL) return HSA_ERR_UNSUPPORTED;
@@ -930,8 +951,7 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   const int rem = (int)(units % sms);
   int pieces = 1;
   if (ws && rem > 0) {
-    pieces = sms / rem;
-    if (pieces > a.n_kv_tiles) pieces = a.n_kv_tiles;
+    pieces = tail_pieces(rem, sms, a.n_kv_tiles);
     const size_t need = (size_t)rem * pieces * (kQT * kBM) * ((size_t)D * 4 + 8);
     if (pieces < 2 || need > ws_bytes || (reinterpret_cast<uintptr_t>(ws) & 15)) pieces = 1;
   }
