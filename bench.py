@@ -220,7 +220,6 @@ def run_hsa(args, dist, rank, world, local_rank):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     n_of = {it: hsa.hsa_active_count(budgets, L.counts, T, it, w.window_pct) for it in L.iters}
-    launches_per_step = 14 + 5 * len(L.iters)
 
     kinds = ("partition", "active", "gather", "scatter", "attention", "euler")
 
@@ -261,6 +260,7 @@ def run_hsa(args, dist, rank, world, local_rank):
 
     barrier(dist)
     torch.cuda.synchronize()
+    launches0 = hsa.hsa_launch_count()
     with ClockSampler(local_rank) as clocks:
         for _ in range(args.steps):
             flush.zero_()                       # L2 flush, outside the step's events
@@ -270,6 +270,7 @@ def run_hsa(args, dist, rank, world, local_rank):
             s1.record(stream)
             step_events.append((s0, s1))
         torch.cuda.synchronize()
+    launches = hsa.hsa_launch_count() - launches0       # this library's kernels only
     barrier(dist)
     step_ms = [a.elapsed_time(b) for a, b in step_events]
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
@@ -315,7 +316,7 @@ def run_hsa(args, dist, rank, world, local_rank):
                    "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
                    "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
         "kernels": kernels, "roofline": roofline,
-        "gpu_launches": launches_per_step * args.steps,
+        "gpu_launches": launches,
         "clocks": clocks.summary(),
     }
     if not args.no_e2e:
@@ -327,60 +328,127 @@ def run_hsa(args, dist, rank, world, local_rank):
 
 
 def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
-    """Same step through the C ABI with host buffers (pinned), copies timed."""
+    """Same step through the C ABI with host buffers (pinned).  Copies run on
+    their own streams and overlap the kernels: each iteration's inputs are
+    copied in one iteration ahead (double-buffered device buffers), each
+    attention output is copied out as soon as it is ready, and the latent
+    after the step.  Timed from the first host-to-device copy to the last
+    device-to-host copy."""
     w = L.w
     T, budgets = w.T, w.budgets
+    iters = L.iters
     n_max = max(n_of.values())
     pin = lambda t: t.cpu().pin_memory()  # noqa: E731
     h_stat = pin(L.stat)
-    h_q = pin(L.q[:n_max])                      # compact active queries
-    h_kf, h_vf = pin(L.kf[:n_max]), pin(L.vf[:n_max])
+    h_q, h_kf, h_vf = pin(L.q[:n_max]), pin(L.kf[:n_max]), pin(L.vf[:n_max])
     h_vfr = pin(L.v_fresh[:n_max])
-    h_out = torch.empty((n_max, w.H, w.D), dtype=L.out.dtype).pin_memory()
+    h_out = [torch.empty((n_of[it], w.H, w.D), dtype=L.out.dtype).pin_memory() for it in iters]
     h_x = torch.empty_like(L.x, device="cpu").pin_memory()
-    d_q = torch.empty_like(L.q[:n_max])
+    bufs = [dict(q=torch.empty_like(L.q[:n_max]), kf=torch.empty_like(L.kf[:n_max]),
+                 vf=torch.empty_like(L.vf[:n_max]), vfr=torch.empty_like(L.v_fresh[:n_max]))
+            for _ in range(2)]
+    outs = [torch.empty((n_max, w.H, w.D), dtype=L.out.dtype, device=dev) for _ in range(2)]
     ws = torch.empty(hsa.hsa_partition_workspace_bytes(w.N), dtype=torch.uint8, device=dev)
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     h2d = L.stat.numel() * 4
     d2h = h_x.numel() * 4
-    for it in L.iters:
+    for it in iters:
         n = n_of[it]
         h2d += n * w.H * w.D * 2 * 3 + n * w.C * 4
         d2h += n * w.H * w.D * 2
+    ev = lambda: torch.cuda.Event()  # noqa: E731
+    # slot events persist across steps: buffer slot j % 2 is free for the
+    # copy-in of use j once compute of use j - 2 is done (in_free) and its
+    # output buffer once the copy-out of use j - 2 is done (out_free)
+    st = {"j": 0, "in_free": [None, None], "out_free": [None, None], "stat_free": None,
+          "x_free": None}
 
     def step():
-        L.stat.copy_(h_stat, non_blocking=True)
+        j0 = st["j"]
+        loaded = {}
+        with torch.cuda.stream(s_in):
+            if st["stat_free"] is not None:
+                s_in.wait_event(st["stat_free"])
+            L.stat.copy_(h_stat, non_blocking=True)
+            stat_ready = ev()
+            stat_ready.record(s_in)
+
+        def load(k):
+            j = j0 + k
+            b, n = bufs[j % 2], n_of[iters[k]]
+            with torch.cuda.stream(s_in):
+                if st["in_free"][j % 2] is not None:
+                    s_in.wait_event(st["in_free"][j % 2])
+                b["q"][:n].copy_(h_q[:n], non_blocking=True)
+                b["kf"][:n].copy_(h_kf[:n], non_blocking=True)
+                b["vf"][:n].copy_(h_vf[:n], non_blocking=True)
+                b["vfr"][:n].copy_(h_vfr[:n], non_blocking=True)
+                e = ev()
+                e.record(s_in)
+                loaded[k] = e
+
+        load(0)
+        stream.wait_event(stat_ready)
         hsa.hsa_partition(L.stat, T, budgets, L.counts, L.group_of, ws, stream)
-        for it in L.iters:
-            n = n_of[it]
+        st["stat_free"] = ev()
+        st["stat_free"].record(stream)
+        for k, it in enumerate(iters):
+            if k + 1 < len(iters):
+                load(k + 1)
+            j = j0 + k
+            b, n = bufs[j % 2], n_of[it]
             ds = sig[it + 1] - sig[it]
-            d_q[:n].copy_(h_q[:n], non_blocking=True)
-            L.kf[:n].copy_(h_kf[:n], non_blocking=True)
-            L.vf[:n].copy_(h_vf[:n], non_blocking=True)
-            L.v_fresh[:n].copy_(h_vfr[:n], non_blocking=True)
+            stream.wait_event(loaded[k])
+            if st["out_free"][j % 2] is not None:
+                stream.wait_event(st["out_free"][j % 2])
             hsa.hsa_partition_active(L.group_of, T, budgets, it, L.idx, L.pos, w.window_pct,
                                      stream)
             hsa.hsa_gather_active(L.hidden, L.idx, n, L.gathered, stream)
-            hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, n, stream)
-            hsa.hsa_active_attention(d_q, None, n, L.kc, L.vc, L.out, 0.0, L.ws_att, stream)
-            h_out[:n].copy_(L.out[:n], non_blocking=True)
-            hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n, stream)
-        h_x.copy_(L.x, non_blocking=True)
+            hsa.hsa_kv_sync_scatter(L.kc, L.vc, b["kf"], b["vf"], L.idx, n, stream)
+            out = outs[j % 2]
+            hsa.hsa_active_attention(b["q"], None, n, L.kc, L.vc, out, 0.0, L.ws_att, stream)
+            e_att = ev()
+            e_att.record(stream)
+            if k == 0 and st["x_free"] is not None:
+                stream.wait_event(st["x_free"])          # previous latent copied out
+            hsa.hsa_cached_euler(L.x, L.vh, b["vfr"], L.pos, ds, n, stream)
+            st["in_free"][j % 2] = ev()
+            st["in_free"][j % 2].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(e_att)
+                h_out[k].copy_(out[:n], non_blocking=True)
+                st["out_free"][j % 2] = ev()
+                st["out_free"][j % 2].record(s_out)
+        st["j"] = j0 + len(iters)
+        fin = ev()
+        fin.record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(fin)
+            h_x.copy_(L.x, non_blocking=True)
+            st["x_free"] = ev()
+            st["x_free"].record(s_out)
 
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
     barrier(dist)
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
+    a.record(s_in)
+    stream.wait_event(a)
+    s_out.wait_event(a)
     for _ in range(args.steps):
         step()
-    b.record(stream)
+    s_out.wait_stream(stream)
+    s_out.wait_stream(s_in)
+    b.record(s_out)
     torch.cuda.synchronize()
     barrier(dist)
     ms = max_over_ranks(dist, a.elapsed_time(b), dev) / args.steps
     assert hsa.hsa_get_device_error(stream) == 0
     return {"value": world * flops_step / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
-            "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+            "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "copies": "pinned host buffers; inputs copied one iteration ahead on a copy "
+                      "stream, outputs copied back on another, overlapping the kernels"}
 
 
 def profiled_traffic(w):

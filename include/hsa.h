@@ -331,6 +331,12 @@ int hsa_cached_euler_l1rel(float *x, float *v_cache, const float *v_fresh,
  * every stream and thread. */
 int hsa_get_device_error(hsa_stream_t stream);
 
+/* Number of kernels this library has launched in this process, on any device
+ * or stream, since it was loaded (a host-side counter, incremented when a
+ * launch is enqueued; a call that fails its argument checks adds nothing).
+ * Never fails; takes no GPU. */
+unsigned long long hsa_launch_count(void);
+
 #ifdef __cplusplus
 }
 #endif

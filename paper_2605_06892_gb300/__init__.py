@@ -26,7 +26,7 @@ __all__ = [
     "hsa_active_attention", "hsa_active_attention_prefix",
     "hsa_active_attention_workspace_bytes",
     "hsa_cached_euler", "hsa_cached_euler_l1rel",
-    "hsa_get_device_error", "hsa_test_inject_attention_stall",
+    "hsa_get_device_error", "hsa_launch_count", "hsa_test_inject_attention_stall",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -81,6 +81,7 @@ _SIGS = {
     "hsa_cached_euler_l1rel": ([_c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_f, _c_p,
                                 _c_f, _c_p], _c_int),
     "hsa_get_device_error": ([_c_p], _c_int),
+    "hsa_launch_count": ([], ctypes.c_ulonglong),
     "hsa_test_inject_attention_stall": ([_c_int], _c_int),
 }
 
@@ -313,6 +314,11 @@ def hsa_cached_euler_l1rel(x, v_cache, v_fresh, pos, dsigma: float, stat, weight
 def hsa_get_device_error(stream=None) -> int:
     """Status of the device-side checks since the last call (synchronises)."""
     return lib().hsa_get_device_error(_stream(stream))
+
+
+def hsa_launch_count() -> int:
+    """Kernels this library has launched in this process (host counter)."""
+    return int(lib().hsa_launch_count())
 
 
 def hsa_test_inject_attention_stall(mode: int) -> int:

@@ -37,6 +37,10 @@ unsigned *device_error_word() {
   return p;
 }
 
+std::atomic<unsigned long long> g_launches{0};
+
+void count_launches(int n) { g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed); }
+
 int sm_count() {
   const int dev = current_device();
   if (dev < 0) return 1;
@@ -132,4 +136,8 @@ extern "C" int hsa_get_device_error(hsa_stream_t stream) {
   if (bits & hsa::kErrNonfinite) return HSA_ERR_NONFINITE;
   if (bits & hsa::kErrIndex) return HSA_ERR_INDEX;
   return HSA_OK;
+}
+
+extern "C" unsigned long long hsa_launch_count(void) {
+  return hsa::g_launches.load(std::memory_order_relaxed);
 }

@@ -960,10 +960,12 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.ws_o = pieces > 1 ? static_cast<float *>(ws) : nullptr;
   a.ws_ml = pieces > 1 ? a.ws_o + (size_t)rem * pieces * (kQT * kBM) * D : nullptr;
   const long long grid = (long long)a.n_whole + (pieces > 1 ? (long long)rem * pieces : 0);
+  count_launches(1);
   attn_tc_kernel<D><<<(unsigned)grid, kTcThreads, C::kSmem, stream>>>(mk, mv, mk2, mv2, a);
   if (cudaGetLastError() != cudaSuccess) return HSA_ERR_CUDA;
   if (pieces > 1) {
     const long long warps = (long long)rem * (kQT * kBM);
+    count_launches(1);
     attn_combine_kernel<D><<<(unsigned)((warps * 32 + 255) / 256), 256, 0, stream>>>(
         a.ws_o, a.ws_ml, rem, a.n_whole, pieces, a.n_qblocks, n_active, H, a.out);
   }
@@ -977,6 +979,7 @@ int launch_f32(const void *q, const int32_t *q_idx, int n_active, const void *k_
   constexpr int QPB = kF32Threads / (D / 32);
   const int N = rows1 + rows2;
   const dim3 grid((n_active + QPB - 1) / QPB, H);
+  count_launches(1);
   attn_f32_kernel<D><<<grid, kF32Threads, 0, stream>>>(
       static_cast<const float *>(q), q_idx, static_cast<const float *>(k_cache),
       static_cast<const float *>(v_cache), rows1, static_cast<const float *>(k_base),

@@ -23,6 +23,10 @@ unsigned *device_error_word();
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// Adds n to the process-wide count of kernels this library has launched
+// (read through hsa_launch_count); called next to every launch.
+void count_launches(int n);
+
 inline int launch_status() {
   return cudaGetLastError() == cudaSuccess ? HSA_OK : HSA_ERR_CUDA;
 }

@@ -366,6 +366,7 @@ extern "C" int hsa_gather_active(const void *src, size_t row_bytes, int N,
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   const int L = lanes_per_row(vecs);
+  count_launches(1);
   gather_rows_kernel<<<grid_for(n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
       (const uint4 *)src, (uint4 *)dst, idx, n_active, N, (int)vecs, log2i(L), err);
   return launch_status();
@@ -388,6 +389,7 @@ extern "C" int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_f
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   const int L = lanes_per_row(vecs);
+  count_launches(1);
   kv_scatter_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
       (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
       n_active, N, (int)vecs, log2i(L), err);
@@ -414,6 +416,7 @@ extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
   long long blocks = (total + (long long)kThreads * per - 1) / ((long long)kThreads * per);
   const long long cap = (long long)sm_count() * (2048 / kThreads);
   if (blocks > cap) blocks = cap;
+  count_launches(1);
   if (per == kEulerUnroll)
     cached_euler_kernel<kEulerUnroll><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
         (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
@@ -438,6 +441,7 @@ extern "C" int hsa_cached_euler_l1rel(float *x, float *v_cache, const float *v_f
   if (!err) return HSA_ERR_CUDA;
   const int vecs = C / 4;
   const int L = lanes_per_row(vecs);
+  count_launches(1);
   euler_l1rel_kernel<<<grid_for(((long long)N + kL1relRows - 1) / kL1relRows, L), kThreads, 0,
                        (cudaStream_t)stream>>>(
       (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, N, vecs, log2i(L), dsigma,
@@ -476,6 +480,7 @@ extern "C" int hsa_rope_rows(void *x, const int32_t *idx, int n, int H, int D,
   const long long vecs = (long long)H * D / 8;
   if (vecs > (1LL << 30)) return HSA_ERR_UNSUPPORTED;
   const int L = lanes_per_row(vecs);
+  count_launches(1);
   rope_rows_kernel<<<grid_for(n, L), kThreads, 0, (cudaStream_t)stream>>>(
       (uint4 *)x, idx, n, (int)vecs, D, (const float4 *)table, N, log2i(L), err);
   return launch_status();
@@ -496,6 +501,7 @@ extern "C" int hsa_kv_sync_scatter_rope(void *k_cache, void *v_cache, const void
   const long long vecs = (long long)H * D / 8;
   if (vecs > (1LL << 30)) return HSA_ERR_UNSUPPORTED;
   const int L = lanes_per_row(vecs);
+  count_launches(1);
   kv_scatter_rope_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
       (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
       n_active, N, (int)vecs, D, (const float4 *)table, log2i(L), err);

@@ -285,11 +285,15 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
   if (!err) return HSA_ERR_CUDA;
   const int ew_blocks = (int)std::min<long long>((N + kSortThreads - 1) / kSortThreads,
                                                  (long long)sm_count() * 8);
+  count_launches(1);
   radix_key_kernel<<<ew_blocks, kSortThreads, 0, s>>>(stat, N, keys[0], vals[0], err);
   for (int pass = 0; pass < 4; ++pass) {
     const int in = pass & 1, out = in ^ 1;
+    count_launches(1);
     radix_hist_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], N, 8 * pass, hist, L.tiles);
+    count_launches(1);
     radix_scan_kernel<<<1, 1024, 0, s>>>(hist, 256 * L.tiles);
+    count_launches(1);
     radix_scatter_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], vals[in], keys[out], vals[out], N,
                                                      8 * pass, hist, L.tiles);
   }
@@ -300,6 +304,7 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
     gs.count[k] = counts[k];
     r += counts[k];
   }
+  count_launches(1);
   group_assign_kernel<<<ew_blocks, kSortThreads, 0, s>>>(vals[0], N, K, gs, group_of);
   return launch_status();
 }
@@ -329,6 +334,7 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
   cudaStream_t s = (cudaStream_t)stream;
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
+  count_launches(1);
   if (aligned16(group_of))
     active_set_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,
                                                         pos, err);
@@ -485,6 +491,7 @@ extern "C" int hsa_uniform_stat(float *stat, int N, hsa_stream_t stream) {
   if (N == 0) return HSA_OK;
   if (!stat) return HSA_ERR_INVALID_ARG;
   const int blocks = (int)std::min<long long>((N + 255) / 256, (long long)sm_count() * 8);
+  count_launches(1);
   uniform_stat_kernel<<<blocks, 256, 0, (cudaStream_t)stream>>>(stat, N);
   return launch_status();
 }
@@ -495,6 +502,7 @@ extern "C" int hsa_reserve_first_frame(float *stat, int N, int frame_tokens,
   if (frame_tokens == 0) return HSA_OK;
   if (!stat) return HSA_ERR_INVALID_ARG;
   const int blocks = (int)std::min<long long>((frame_tokens + 255) / 256, (long long)sm_count() * 8);
+  count_launches(1);
   reserve_frame_kernel<<<blocks, 256, 0, (cudaStream_t)stream>>>(stat, frame_tokens);
   return launch_status();
 }
@@ -514,6 +522,7 @@ extern "C" int hsa_reorder_tokens(const int32_t *group_of, int N, int n_baseline
   const int blocks = (int)(((long long)N + chunk - 1) / chunk);
   const int M = N - n_baseline;
   cudaStream_t s = (cudaStream_t)stream;
+  count_launches(1);
   if (aligned16(group_of))
     reorder_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, M, (int)chunk, order, where,
                                                          group_new, err);

@@ -95,3 +95,17 @@ def test_rope_table_matches_oracle(hsa):
         a = hsa.hsa_rope_table(grid, D)
         b = oracle.rope_table(grid, D)
         assert torch.allclose(a, b, rtol=0, atol=1e-7)
+
+
+def test_launch_counter_needs_no_gpu(hsa):
+    """The launch counter is host-side: readable without a GPU, and host-only
+    calls and calls that fail their argument checks add nothing."""
+    c0 = hsa.hsa_launch_count()
+    assert isinstance(c0, int) and c0 >= 0
+    hsa.hsa_check_budgets(40, (40, 20), (1, 1), 2)
+    hsa.hsa_window_margin(40, 80)
+    ints = ctypes.c_int * 2
+    # 15 does not divide T = 40: rejected on the host, nothing launched
+    st = hsa.lib().hsa_partition(None, 4, 40, ints(40, 15), ints(2, 2), 2, None, None, 0, None)
+    assert st < 0
+    assert hsa.hsa_launch_count() == c0
