@@ -24,8 +24,8 @@
 // redone with its exact maximum (and O rescaled in TMEM).  The final division
 // by the running sum makes the result exact whatever reference was used.
 // Registers: the block launches at 168 per thread; the first warpgroup then
-// gives registers back (setmaxnreg.dec to 88) and the two softmax warpgroups
-// take them (setmaxnreg.inc to 208): 128*88 + 256*208 = 384*168.
+// gives registers back (setmaxnreg.dec to 96) and the two softmax warpgroups
+// take them (setmaxnreg.inc to 200): 128*96 + 256*200 <= 384*168.
 // Every mbarrier wait is bounded in time; on a timeout the kernel records
 // HSA_ERR_TIMEOUT, stops issuing work, drains its own copies and MMAs, frees
 // TMEM and returns.
@@ -277,8 +277,8 @@ constexpr int kQT = 2;           // Q tiles per CTA
 constexpr int kBN = 128;         // keys per K/V tile
 constexpr int kTcThreads = 384;  // 12 warps = 3 warpgroups
 constexpr int kLaunchRegs = 168;         // registers per thread at launch
-constexpr int kRegsLow = 88;             // producer / MMA warpgroup
-constexpr int kRegsHigh = 208;           // softmax warpgroups
+constexpr int kRegsLow = 96;             // producer / MMA warpgroup
+constexpr int kRegsHigh = 200;           // softmax warpgroups
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kTcThreads * kLaunchRegs,
               "register split exceeds the launch allocation");
 constexpr int kTmemCols = 512;
@@ -466,7 +466,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     }
     for (int t = 0; t < kQT; ++t) {
       mbar_init(&bar_s[t], 1);
-      mbar_init(&bar_p[t], kBM);
+      mbar_init(&bar_p[t], kBM / 32);      // one arrive per softmax warp
     }
     mbar_init(&bar_o, 1);
     abort_flag = 0;
@@ -662,7 +662,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         softmax_tile<D, true>(tS, tO, valid, j == 0, sl2, m_run, l_run);
       tmem_wait_st();
       fence_before();
-      if (!(a.inject_stall == 1 && t == 0 && j == 0)) mbar_arrive(&bar_p[t]);
+      __syncwarp();
+      if (lane == 0 && !(a.inject_stall == 1 && t == 0 && j == 0)) mbar_arrive(&bar_p[t]);
     }
     if (ok && wk.piece >= 0 && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
       // Piece of a split unit: unnormalised O, maximum and sum, for the combine.
