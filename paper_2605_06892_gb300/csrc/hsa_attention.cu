@@ -66,17 +66,6 @@ __device__ __forceinline__ void mbar_arrive(uint64_t *b) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(b)) : "memory");
 }
 
-__device__ __forceinline__ bool mbar_test(uint64_t *b, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(smem_addr(b)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
 // Non-blocking test of phase `parity` (never suspends the thread).
 __device__ __forceinline__ bool mbar_peek(uint64_t *b, uint32_t parity) {
   uint32_t ok;
@@ -108,13 +97,18 @@ constexpr long long kWaitCycles = 2000000000LL;
 
 // Bounded wait on phase `parity` of barrier b.  Gives up when the time runs
 // out (records the timeout and raises the CTA's abort flag) or, if
-// `honor_abort`, as soon as another role has raised the abort flag.
+// `honor_abort`, as soon as another role has raised the abort flag.  The
+// first test is a non-blocking test_wait: try_wait costs a few hundred clocks
+// even on a completed phase, which on the MMA issuer's path leaves the tensor
+// pipe idle.  `spin` keeps testing with test_wait (the MMA issuer, which must
+// resume at once); otherwise the thread suspends in try_wait between tests.
 __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
-                                          unsigned *err, bool honor_abort = true) {
-  if (mbar_test(b, parity)) return true;
+                                          unsigned *err, bool honor_abort = true,
+                                          bool spin = false) {
+  if (mbar_peek(b, parity)) return true;
   const long long t0 = clock64();
   while (true) {
-    if (mbar_test_suspend(b, parity)) return true;
+    if (spin ? mbar_peek(b, parity) : mbar_test_suspend(b, parity)) return true;
     if (honor_abort && *abort_flag) return false;
     if (clock64() - t0 > kWaitCycles) {
       set_error(err, kErrTimeout);
@@ -545,7 +539,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         const uint32_t q_base = smem_addr(sQ);
         const uint32_t kv_base = smem_addr(sKV);
         auto wait_full = [&](int L) {
-          return mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err);
+          return mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err,
+                           true, true);
         };
         // Descriptors differ only in their start-address field (bits 0-13,
         // address >> 4), so each MMA adds a constant to a base descriptor.
@@ -597,7 +592,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
           const int Lv = 2 * j + 1, Lk = 2 * j + 2;
           const bool more = j + 1 < nT;
           if (!rdy_v && !(ok = wait_full(Lv))) break;
-          if (!rdy_p0 && !(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err))) break;
+          if (!rdy_p0 && !(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err, true, true))) break;
           fence_after();
           issue_o(0, Lv, j > 0, [&] { rdy_k = more && full_ready(Lk); });
           if (more) {
@@ -608,7 +603,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
           } else {
             rdy_p1 = false;
           }
-          if (!rdy_p1 && !(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err))) break;
+          if (!rdy_p1 && !(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err, true, true))) break;
           fence_after();
           if (more) {
             issue_o(1, Lv, j > 0, [] {});
