@@ -334,7 +334,8 @@ int hsa_get_device_error(hsa_stream_t stream);
 /* Number of kernels this library has launched in this process, on any device
  * or stream, since it was loaded (a host-side counter, incremented when a
  * launch is enqueued; a call that fails its argument checks adds nothing).
- * Never fails; takes no GPU. */
+ * A call captured into a CUDA graph counts once, at capture; replays of the
+ * graph are not counted.  Never fails; takes no GPU. */
 unsigned long long hsa_launch_count(void);
 
 #ifdef __cplusplus
