@@ -549,10 +549,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         const uint64_t dv0 = sdesc(kv_base, kBN * 128, 1024);
         constexpr uint32_t kTile16 = C::kTileBytes >> 4;
         // The tensor pipe queues only a few MMAs, so the issuing thread must
-        // not stop with an empty queue.  Each group of eight MMAs therefore
-        // issues six, then `peek`s (non-blocking) the barriers the next group
+        // not stop with an empty queue.  A group of eight MMAs therefore
+        // issues six, then `peek`s (non-blocking) the barriers a later group
         // needs while the last queued MMAs still run, then issues the last two;
-        // a barrier found complete needs no blocking wait afterwards.
+        // a barrier found complete needs no blocking wait afterwards.  The
+        // peeks for the next key tile's V and P_0 sit in the O_1 group rather
+        // than the S_1 group: an S group's operand reads fill the shared-memory
+        // bandwidth, and a barrier test issued then comes back late.
         // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
         auto issue_s = [&](int t, int L, auto peek) {
           const uint64_t dq = dq0 + t * kTile16;
@@ -606,12 +609,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
           if (!rdy_p1 && !(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err, true, true))) break;
           fence_after();
           if (more) {
-            issue_o(1, Lv, j > 0, [] {});
-            mma_commit(&bar_empty[Lv % C::kStages]);
-            issue_s(1, Lk, [&] {
+            issue_o(1, Lv, j > 0, [&] {
               rdy_v = full_ready(Lv + 2);
               rdy_p0 = mbar_peek(&bar_p[0], (j + 1) & 1);
             });
+            mma_commit(&bar_empty[Lv % C::kStages]);
+            issue_s(1, Lk, [] {});
             mma_commit(&bar_s[1]);
             mma_commit(&bar_empty[Lk % C::kStages]);
           } else {
