@@ -294,9 +294,29 @@ def run_hsa(args, dist, rank, world, local_rank):
     for k in ("gather", "scatter", "euler", "active"):
         gbs = bytes_step[k] / (kern_ms[k] * 1e-3) / 1e9
         kernels[k] = {"ms": kern_ms[k], "gbs": gbs, "frac_hbm": gbs / peaks["hbm_gbs"]}
+    # per-iteration layer time (the five kernels of each iteration), and the
+    # same iteration with every token active (i = 0 activates every group):
+    # the dense all-token baseline, through the same kernels
+    n_it = len(L.iters)
+    it_ms = [0.0] * n_it
+    att_ms = [0.0] * n_it
+    for kind in ("active", "gather", "scatter", "attention", "euler"):
+        for e, (a, b) in enumerate(per_kernel[kind]):
+            t = a.elapsed_time(b) / args.steps
+            it_ms[e % n_it] += t
+            if kind == "attention":
+                att_ms[e % n_it] += t
+    dense = dense_iteration(args, hsa, L, sig, flush, ws_att, stream)
     per_iter = {}
-    for it in L.iters:
-        per_iter[str(it)] = {"n_active": n_of[it], "frac": n_of[it] / w.N}
+    for m, it in enumerate(L.iters):
+        per_iter[str(it)] = {"n_active": n_of[it], "frac": n_of[it] / w.N, "ms": it_ms[m],
+                             "attention_ms": att_ms[m], "vs_dense": it_ms[m] / dense["ms"]}
+    dense_baseline = {
+        "iteration_ms": dense["ms"], "attention_ms": dense["attention_ms"],
+        "step_ms_all_dense": n_it * dense["ms"] + kern_ms["partition"],
+        "step_vs_all_dense": ms_per_step / (n_it * dense["ms"] + kern_ms["partition"]),
+        "what": f"{n_it} iterations with every token active (same kernels, |A| = N), "
+                "against the measured step; L2 flushed before each dense iteration"}
 
     att_tflops = kernels["attention"]["tflops"]
     roofline = {"bound": "tensor", "achieved": att_tflops, "peak": peaks["bf16_tflops"],
@@ -315,7 +335,7 @@ def run_hsa(args, dist, rank, world, local_rank):
                    "per_iteration": per_iter, "parallelism": f"replicas x{world}",
                    "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
                    "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
-        "kernels": kernels, "roofline": roofline,
+        "kernels": kernels, "roofline": roofline, "dense_baseline": dense_baseline,
         "gpu_launches": launches,
         "clocks": clocks.summary(),
     }
@@ -325,6 +345,38 @@ def run_hsa(args, dist, rank, world, local_rank):
         line["cpu_baseline"] = cpu_baseline(w, L)
     if rank == 0:
         print(json.dumps(line), flush=True)
+
+
+def dense_iteration(args, hsa, L, sig, flush, ws_att, stream, reps=None):
+    """Time one HSA iteration with every token active (iteration 0 of the
+    schedule activates every group): active set, gather, KV-sync scatter,
+    attention over all N queries, cached Euler.  L2 flushed before each rep;
+    outside the benchmark's timed region."""
+    w = L.w
+    T, budgets = w.T, w.budgets
+    reps = reps or max(3, min(args.steps, 10))
+    ds = sig[1] - sig[0]
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    tot, att = [], []
+    for r in range(reps + 1):
+        flush.zero_()
+        a, b, c, d = ev(), ev(), ev(), ev()
+        a.record(stream)
+        hsa.hsa_partition_active(L.group_of, T, budgets, 0, L.idx, L.pos, w.window_pct, stream)
+        hsa.hsa_gather_active(L.hidden, L.idx, w.N, L.gathered, stream)
+        hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, w.N, stream)
+        b.record(stream)
+        hsa.hsa_active_attention(L.q, L.idx, w.N, L.kc, L.vc, L.out, 0.0, ws_att, stream)
+        c.record(stream)
+        hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, w.N, stream)
+        d.record(stream)
+        if r > 0:                                  # the first rep is a warm-up
+            tot.append((a, d))
+            att.append((b, c))
+    torch.cuda.synchronize()
+    assert hsa.hsa_get_device_error(stream) == 0
+    return {"ms": sum(x.elapsed_time(y) for x, y in tot) / reps,
+            "attention_ms": sum(x.elapsed_time(y) for x, y in att) / reps}
 
 
 def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
