@@ -16,11 +16,10 @@ extern "C" {
 #endif
 
 /* mode 0: normal operation (default).
- * mode 1: in every bf16 hsa_active_attention launch that follows, the softmax
- *         of the first query tile of each CTA never releases its first block
- *         of probabilities, so the tensor-core issuer's bounded wait runs out;
- *         the call then reports HSA_ERR_TIMEOUT through hsa_get_device_error
- *         and its output is unspecified.
+ * mode 1: in every bf16 hsa_active_attention launch that follows, each CTA
+ *         never loads its first value tile, so the bounded wait for it runs
+ *         out; the call then reports HSA_ERR_TIMEOUT through
+ *         hsa_get_device_error and its output is unspecified.
  * Process-wide, host side only; returns the previous mode, or
  * HSA_ERR_INVALID_ARG (-1) for an unknown mode. */
 int hsa_test_inject_attention_stall(int mode);

@@ -323,6 +323,6 @@ def hsa_launch_count() -> int:
 
 def hsa_test_inject_attention_stall(mode: int) -> int:
     """Test hook (include/hsa_test.h): mode 1 makes following bf16 attention
-    launches withhold one internal signal so their bounded wait runs out and
-    HSA_ERR_TIMEOUT is reported; mode 0 restores normal operation."""
+    launches never load their first value tile, so the bounded wait for it runs
+    out and HSA_ERR_TIMEOUT is reported; mode 0 restores normal operation."""
     return _check(lib().hsa_test_inject_attention_stall(mode), "hsa_test_inject_attention_stall")

@@ -62,10 +62,6 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
                : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(b)) : "memory");
-}
-
 // Non-blocking test of phase `parity` (never suspends the thread).
 __device__ __forceinline__ bool mbar_peek(uint64_t *b, uint32_t parity) {
   uint32_t ok;
@@ -98,17 +94,14 @@ constexpr long long kWaitCycles = 2000000000LL;
 // Bounded wait on phase `parity` of barrier b.  Gives up when the time runs
 // out (records the timeout and raises the CTA's abort flag) or, if
 // `honor_abort`, as soon as another role has raised the abort flag.  The
-// first test is a non-blocking test_wait: try_wait costs a few hundred clocks
-// even on a completed phase, which on the MMA issuer's path leaves the tensor
-// pipe idle.  `spin` keeps testing with test_wait (the MMA issuer, which must
-// resume at once); otherwise the thread suspends in try_wait between tests.
+// first test is a non-blocking test_wait (a try_wait costs far more even on a
+// completed phase); between tests the thread suspends in try_wait.
 __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_flag,
-                                          unsigned *err, bool honor_abort = true,
-                                          bool spin = false) {
+                                          unsigned *err, bool honor_abort = true) {
   if (mbar_peek(b, parity)) return true;
   const long long t0 = clock64();
   while (true) {
-    if (spin ? mbar_peek(b, parity) : mbar_test_suspend(b, parity)) return true;
+    if (mbar_test_suspend(b, parity)) return true;
     if (honor_abort && *abort_flag) return false;
     if (clock64() - t0 > kWaitCycles) {
       set_error(err, kErrTimeout);
@@ -253,6 +246,7 @@ __device__ __forceinline__ void named_barrier_sync(int id, int threads) {
   asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
+
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -276,6 +270,16 @@ constexpr int kRegsHigh = 200;           // softmax warpgroups
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kTcThreads * kLaunchRegs,
               "register split exceeds the launch allocation");
 constexpr int kTmemCols = 512;
+// Named barriers (hardware, not in shared memory): 1 = teardown of the whole
+// CTA; kBarP0 + t = P of Q tile t is in TMEM (its 128 softmax threads and the
+// issuing warp meet); kBarKV0 + s = the K/V tile in ring slot s has landed
+// (the K/V watcher warp and the issuing warp meet).  Every party syncs
+// (a rendezvous, never a lone arrive) once per hand-off in the same order, so
+// no party can run a whole round ahead and the barrier instances always pair
+// up, also after a failed wait.
+constexpr int kBarTeardown = 1;
+constexpr int kBarP0 = 2;
+constexpr int kBarKV0 = 4;
 
 template <int D>
 struct TcCfg {
@@ -294,7 +298,7 @@ struct TcArgs {
   int n_active, N, H, q_rows, n_kv_tiles;
   int rows1, rows2, tiles1;   // key sources: rows1 cache rows, then rows2 rows
   float scale_log2;
-  int inject_stall;   // test hook (hsa_test.h): 1 = tile 0 withholds its first P
+  int inject_stall;   // test hook (hsa_test.h): 1 = the first V tile is never loaded
   // Work split.  CTA b < n_whole owns unit b (head b / n_qblocks, query block
   // b % n_qblocks) over all key tiles.  Every later CTA owns one of `pieces`
   // key ranges of a tail unit and writes its unnormalised O, running maximum
@@ -442,7 +446,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   uint8_t *sQ = sm;
   uint8_t *sKV = sm + kQT * C::kTileBytes;
   __shared__ __align__(8) uint64_t bar_full[C::kStages], bar_empty[C::kStages];
-  __shared__ __align__(8) uint64_t bar_s[kQT], bar_p[kQT], bar_o;
+  __shared__ __align__(8) uint64_t bar_s[kQT], bar_o;
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
 
@@ -458,10 +462,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_empty[s], 1);
     }
-    for (int t = 0; t < kQT; ++t) {
-      mbar_init(&bar_s[t], 1);
-      mbar_init(&bar_p[t], kBM / 32);      // one arrive per softmax warp
-    }
+    for (int t = 0; t < kQT; ++t) mbar_init(&bar_s[t], 1);
     mbar_init(&bar_o, 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -505,15 +506,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   // The warpgroups' code paths never rejoin below: each ends with its own
   // teardown on named barrier 1, so each path is compiled for its own
   // register budget.
+  static_assert(kBarKV0 + C::kStages <= 16, "named barrier ids");
   if (warp < 4) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
     if (warp == 0) {
       // ------------------------------------------------ TMA producer
       if (lane == 0) {
         int issued = 0;
+        const int withheld = a.inject_stall == 1 ? 1 : -1;   // test hook
         for (int L = 0; L < 2 * nT; ++L) {
           const int slot = L % C::kStages, use = L / C::kStages;
           if (use > 0 && !mbar_wait(&bar_empty[slot], (use - 1) & 1, &abort_flag, a.err)) break;
+          if (L == withheld) continue;
           mbar_expect_tx(&bar_full[slot], C::kTileBytes);
           const int jg = j0 + (L >> 1);                   // global key tile
           const bool second = jg >= a.tiles1;
@@ -526,111 +530,121 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
             tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, y);
           issued = L + 1;
         }
-        // Drain: every issued copy has landed before the CTA may exit.
+        // Drain: every issued copy has landed before the CTA may exit.  A
+        // slot is only refilled once its previous tile was consumed, so the
+        // copies in flight are among the last kStages issued.
         for (int L = issued > C::kStages ? issued - C::kStages : 0; L < issued; ++L)
-          mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err, false);
+          if (L != withheld)
+            mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err, false);
       }
       __syncwarp();
       } else if (warp == 1) {
       // ------------------------------------------------ MMA issuer
-      if (lane == 0) {
-        constexpr uint32_t kIdS = idesc_bf16(kBM, kBN, 0);
-        constexpr uint32_t kIdO = idesc_bf16(kBM, D, 1);
-        const uint32_t q_base = smem_addr(sQ);
-        const uint32_t kv_base = smem_addr(sKV);
-        auto wait_full = [&](int L) {
-          return mbar_wait(&bar_full[L % C::kStages], (L / C::kStages) & 1, &abort_flag, a.err,
-                           true, true);
-        };
-        // Descriptors differ only in their start-address field (bits 0-13,
-        // address >> 4), so each MMA adds a constant to a base descriptor.
-        const uint64_t dq0 = sdesc(q_base, 16, 1024);
-        const uint64_t dk0 = sdesc(kv_base, 16, 1024);
-        const uint64_t dv0 = sdesc(kv_base, kBN * 128, 1024);
-        constexpr uint32_t kTile16 = C::kTileBytes >> 4;
-        // The tensor pipe queues only a few MMAs, so the issuing thread must
-        // not stop with an empty queue.  A group of eight MMAs therefore
-        // issues six, then `peek`s (non-blocking) the barriers a later group
-        // needs while the last queued MMAs still run, then issues the last two;
-        // a barrier found complete needs no blocking wait afterwards.  The
-        // peeks for the next key tile's V and P_0 sit in the O_1 group rather
-        // than the S_1 group: an S group's operand reads fill the shared-memory
-        // bandwidth, and a barrier test issued then comes back late.
-        // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
-        auto issue_s = [&](int t, int L, auto peek) {
-          const uint64_t dq = dq0 + t * kTile16;
-          const uint64_t dk = dk0 + (L % C::kStages) * kTile16;
-          const uint32_t ts = tmem + 128 * t;
+      // The whole warp walks the schedule so that it can take part in the
+      // named-barrier hand-offs; lane 0 issues the MMAs and commits.  The
+      // tensor pipe takes a new MMA only about when it starts it, so every
+      // pause of the issuing thread between MMAs idles the tensor core.  An
+      // mbarrier test on this path costs about a hundred clocks while an S
+      // group's operand reads fill the shared-memory bandwidth; a named
+      // barrier whose other parties have already arrived costs far less.
+      // So the issuer waits on named barriers only: kBarKV0 + slot (the K/V
+      // watcher saw the tile land) and kBarP0 + t (the softmax of Q tile t
+      // stored P).  Every party meets it exactly once per hand-off whatever
+      // happens, so each sync completes; after an abort the warp keeps its
+      // syncs but issues nothing more.
+      const bool leader = lane == 0;
+      constexpr uint32_t kIdS = idesc_bf16(kBM, kBN, 0);
+      constexpr uint32_t kIdO = idesc_bf16(kBM, D, 1);
+      const uint32_t q_base = smem_addr(sQ);
+      const uint32_t kv_base = smem_addr(sKV);
+      // Descriptors differ only in their start-address field (bits 0-13,
+      // address >> 4), so each MMA adds a constant to a base descriptor.
+      const uint64_t dq0 = sdesc(q_base, 16, 1024);
+      const uint64_t dk0 = sdesc(kv_base, 16, 1024);
+      const uint64_t dv0 = sdesc(kv_base, kBN * 128, 1024);
+      constexpr uint32_t kTile16 = C::kTileBytes >> 4;
+      // S_t = Q_t K^T: K = D in steps of 16 (32 bytes inside a 128-byte chunk).
+      auto issue_s = [&](int t, int L) {
+        const uint64_t dq = dq0 + t * kTile16;
+        const uint64_t dk = dk0 + (L % C::kStages) * kTile16;
+        const uint32_t ts = tmem + 128 * t;
 #pragma unroll
-          for (int k = 0; k < D / 16; ++k) {
-            if (k == D / 16 - 2) peek();
-            const uint32_t off = ((k >> 2) * (kBM * 128) + (k & 3) * 32) >> 4;
-            mma_ss(ts, dq + off, dk + off, kIdS, k > 0);
-          }
-        };
-        // O_t += P_t V: P in TMEM (bf16 pairs in the S_t columns), V MN-major.
-        auto issue_o = [&](int t, int L, bool acc, auto peek) {
-          const uint64_t dv = dv0 + (L % C::kStages) * kTile16;
-          const uint32_t to = tmem + C::kOCol0 + D * t, tp = tmem + 128 * t;
-#pragma unroll
-          for (int k = 0; k < kBN / 16; ++k) {
-            if (k == kBN / 16 - 2) peek();
-            mma_ts(to, tp + 8 * k, dv + ((k * 2048) >> 4), kIdO, (acc || k > 0) ? 1u : 0u);
-          }
-        };
-        auto full_ready = [&](int L) {
-          return mbar_peek(&bar_full[L % C::kStages], (L / C::kStages) & 1);
-        };
-        bool ok = wait_full(0);
-        bool rdy_v = false, rdy_k = false, rdy_p0 = false, rdy_p1 = false;
-        if (ok) {
-          fence_after();
-          issue_s(0, 0, [] {});
-          mma_commit(&bar_s[0]);
-          issue_s(1, 0, [&] { rdy_v = nT > 0 && full_ready(1); });
-          mma_commit(&bar_s[1]);
-          mma_commit(&bar_empty[0]);
+        for (int k = 0; k < D / 16; ++k) {
+          const uint32_t off = ((k >> 2) * (kBM * 128) + (k & 3) * 32) >> 4;
+          mma_ss(ts, dq + off, dk + off, kIdS, k > 0);
         }
-        for (int j = 0; ok && j < nT; ++j) {
-          const int Lv = 2 * j + 1, Lk = 2 * j + 2;
-          const bool more = j + 1 < nT;
-          if (!rdy_v && !(ok = wait_full(Lv))) break;
-          if (!rdy_p0 && !(ok = mbar_wait(&bar_p[0], j & 1, &abort_flag, a.err, true, true))) break;
-          fence_after();
-          issue_o(0, Lv, j > 0, [&] { rdy_k = more && full_ready(Lk); });
-          if (more) {
-            if (!rdy_k && !(ok = wait_full(Lk))) break;
-            fence_after();
-            issue_s(0, Lk, [&] { rdy_p1 = mbar_peek(&bar_p[1], j & 1); });
+      };
+      // O_t += P_t V: P in TMEM (bf16 pairs in the S_t columns), V MN-major.
+      auto issue_o = [&](int t, int L, bool acc) {
+        const uint64_t dv = dv0 + (L % C::kStages) * kTile16;
+        const uint32_t to = tmem + C::kOCol0 + D * t, tp = tmem + 128 * t;
+#pragma unroll
+        for (int k = 0; k < kBN / 16; ++k)
+          mma_ts(to, tp + 8 * k, dv + ((k * 2048) >> 4), kIdO, (acc || k > 0) ? 1u : 0u);
+      };
+      auto kv_ready = [&](int L) {
+        named_barrier_sync(kBarKV0 + L % C::kStages, 64);
+        fence_after();
+      };
+      auto p_ready = [&](int t) {
+        named_barrier_sync(kBarP0 + t, kBM + 32);
+        fence_after();
+      };
+      kv_ready(0);
+      if (leader && !abort_flag) {
+        issue_s(0, 0);
+        mma_commit(&bar_s[0]);
+        issue_s(1, 0);
+        mma_commit(&bar_s[1]);
+        mma_commit(&bar_empty[0]);
+      }
+      for (int j = 0; j < nT; ++j) {
+        const int Lv = 2 * j + 1, Lk = 2 * j + 2;
+        const bool more = j + 1 < nT;
+        kv_ready(Lv);
+        p_ready(0);
+        const bool go = leader && !abort_flag;
+        if (go) issue_o(0, Lv, j > 0);
+        if (more) {
+          kv_ready(Lk);
+          if (go) {
+            issue_s(0, Lk);
             mma_commit(&bar_s[0]);
-          } else {
-            rdy_p1 = false;
           }
-          if (!rdy_p1 && !(ok = mbar_wait(&bar_p[1], j & 1, &abort_flag, a.err, true, true))) break;
-          fence_after();
+        }
+        p_ready(1);
+        if (go) {
+          issue_o(1, Lv, j > 0);
+          mma_commit(&bar_empty[Lv % C::kStages]);
           if (more) {
-            issue_o(1, Lv, j > 0, [&] {
-              rdy_v = full_ready(Lv + 2);
-              rdy_p0 = mbar_peek(&bar_p[0], (j + 1) & 1);
-            });
-            mma_commit(&bar_empty[Lv % C::kStages]);
-            issue_s(1, Lk, [] {});
+            issue_s(1, Lk);
             mma_commit(&bar_s[1]);
             mma_commit(&bar_empty[Lk % C::kStages]);
-          } else {
-            issue_o(1, Lv, j > 0, [] {});
-            mma_commit(&bar_empty[Lv % C::kStages]);
           }
         }
-        // Completes once every MMA issued above has finished (also on abort),
-        // so TMEM is quiet before it is freed.
+      }
+      if (leader) {
+        // Completes once every MMA issued above has finished (also on
+        // abort), so TMEM is quiet before it is freed.
         mma_commit(&bar_o);
         mbar_wait(&bar_o, 0, &abort_flag, a.err, false);
       }
       __syncwarp();
+    } else if (warp == 2) {
+      // ------------------------------------------------ K/V watcher
+      // Waits (bounded) for each K/V tile to land and meets the issuer on
+      // the slot's named barrier.  It meets it once per tile even after a
+      // failed wait, so the issuer never waits forever.
+      bool live = true;
+      for (int L = 0; L < 2 * nT; ++L) {
+        if (live)
+          live = __all_sync(0xffffffffu, mbar_wait(&bar_full[L % C::kStages],
+                                                   (L / C::kStages) & 1, &abort_flag, a.err));
+        named_barrier_sync(kBarKV0 + L % C::kStages, 64);
+      }
     }
     fence_before();
-    named_barrier_sync(1, kTcThreads);
+    named_barrier_sync(kBarTeardown, kTcThreads);
     if (warp == 1) {
       fence_after();
       asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
@@ -648,20 +662,26 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     const uint32_t tO = tmem + lane_off + C::kOCol0 + D * t;
     const float sl2 = a.scale_log2;
     float m_run = -INFINITY, l_run = 0.f;
+    // `ok` stays warp-uniform (the tile code votes across the warp).  After
+    // a failed wait the warp does no more work but still meets the issuer for
+    // every P, so the issuing warp's named-barrier syncs all complete.
+    // Meeting (rather than arriving) costs nothing: S_t(j+1) is issued only
+    // after the issuer has passed this meeting for P_t(j).
     bool ok = true;
     for (int j = 0; j < nT; ++j) {
-      if (!(ok = mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err))) break;
-      fence_after();
-      const int jg = j0 + j;                       // keys of this tile that exist
-      const int valid = jg < a.tiles1 ? a.rows1 - jg * kBN : a.rows2 - (jg - a.tiles1) * kBN;
-      if (valid >= kBN)
-        softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
-      else
-        softmax_tile<D, true>(tS, tO, valid, j == 0, sl2, m_run, l_run);
-      tmem_wait_st();
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err));
+      if (ok) {
+        fence_after();
+        const int jg = j0 + j;                     // keys of this tile that exist
+        const int valid = jg < a.tiles1 ? a.rows1 - jg * kBN : a.rows2 - (jg - a.tiles1) * kBN;
+        if (valid >= kBN)
+          softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
+        else
+          softmax_tile<D, true>(tS, tO, valid, j == 0, sl2, m_run, l_run);
+        tmem_wait_st();
+      }
       fence_before();
-      __syncwarp();
-      if (lane == 0 && !(a.inject_stall == 1 && t == 0 && j == 0)) mbar_arrive(&bar_p[t]);
+      named_barrier_sync(kBarP0 + t, kBM + 32);
     }
     if (ok && wk.piece >= 0 && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
       // Piece of a split unit: unnormalised O, maximum and sum, for the combine.
@@ -704,7 +724,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       }
     }
     fence_before();
-    named_barrier_sync(1, kTcThreads);
+    named_barrier_sync(kBarTeardown, kTcThreads);
   }
 }
 

@@ -1,6 +1,6 @@
 """Failure detection on the GPU without a fault: the attention kernel's
-bounded pipeline wait is made to run out (one internal signal withheld through
-the test hook), the call reports HSA_ERR_TIMEOUT through the device error
+bounded pipeline wait is made to run out (through the test hook the first
+value tile is never loaded), the call reports HSA_ERR_TIMEOUT through the device error
 word, and the same CUDA context then runs a normal call correctly."""
 import time
 
