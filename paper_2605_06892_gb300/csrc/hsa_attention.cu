@@ -62,6 +62,10 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
                : "memory");
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(b)) : "memory");
+}
+
 // Non-blocking test of phase `parity` (never suspends the thread).
 __device__ __forceinline__ bool mbar_peek(uint64_t *b, uint32_t parity) {
   uint32_t ok;
@@ -285,7 +289,7 @@ template <int D>
 struct TcCfg {
   static constexpr int kTileBytes = kBM * D * 2;            // one Q, K or V tile
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
-  static constexpr int kStages = D == 128 ? 4 : 8;          // K/V ring slots
+  static constexpr int kStages = D == 128 ? 5 : 8;          // K/V ring slots
   static constexpr int kSmem = (kQT + kStages) * kTileBytes + 1024;
   static constexpr int kOCol0 = 256;                        // O_t at kOCol0 + t*D
 };
@@ -596,7 +600,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         mma_commit(&bar_s[0]);
         issue_s(1, 0);
         mma_commit(&bar_s[1]);
-        mma_commit(&bar_empty[0]);
       }
       for (int j = 0; j < nT; ++j) {
         const int Lv = 2 * j + 1, Lk = 2 * j + 2;
@@ -615,11 +618,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         p_ready(1);
         if (go) {
           issue_o(1, Lv, j > 0);
-          mma_commit(&bar_empty[Lv % C::kStages]);
           if (more) {
             issue_s(1, Lk);
             mma_commit(&bar_s[1]);
-            mma_commit(&bar_empty[Lk % C::kStages]);
           }
         }
       }
@@ -634,13 +635,32 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       // ------------------------------------------------ K/V watcher
       // Waits (bounded) for each K/V tile to land and meets the issuer on
       // the slot's named barrier.  It meets it once per tile even after a
-      // failed wait, so the issuer never waits forever.
+      // failed wait, so the issuer never waits forever.  It also gives slots
+      // back to the producer, so the issuer commits nothing for them: once
+      // S_1 of key tile j has completed (the tensor core runs its MMAs in
+      // order), K_j and V_(j-1) have been read by every MMA that uses them.
+      // It waits for that right after meeting the issuer for V_j: S_1 of key
+      // tile j+1 needs K_(j+1), which it has not handed over yet, so the
+      // phase it waits for is never overtaken.  After a failure it gives
+      // nothing back, so no slot is refilled while a copy into it may still
+      // be in flight.
       bool live = true;
+      auto give_back = [&](int L) {
+        if (lane == 0) mbar_arrive(&bar_empty[L % C::kStages]);
+      };
       for (int L = 0; L < 2 * nT; ++L) {
         if (live)
           live = __all_sync(0xffffffffu, mbar_wait(&bar_full[L % C::kStages],
                                                    (L / C::kStages) & 1, &abort_flag, a.err));
         named_barrier_sync(kBarKV0 + L % C::kStages, 64);
+        if ((L & 1) && live) {                     // L = V_j, j = L / 2
+          const int j = L >> 1;
+          live = __all_sync(0xffffffffu, mbar_wait(&bar_s[1], j & 1, &abort_flag, a.err));
+          if (live) {
+            give_back(2 * j);                      // K_j
+            if (j > 0) give_back(2 * j - 1);       // V_(j-1)
+          }
+        }
       }
     }
     fence_before();
