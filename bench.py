@@ -27,6 +27,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -506,19 +507,28 @@ def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
                       "stream, outputs copied back on another, overlapping the kernels"}
 
 
+def code_digest(text: str) -> str:
+    """Digest of a CUDA source with its comments and whitespace removed, so
+    that an edit to comments alone does not invalidate a profile."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    text = " ".join(text.split())
+    return hashlib.sha256(text.encode()).hexdigest()[:16]
+
+
 def profiled_traffic(w):
     """DRAM bytes per attention launch from the committed ncu summary, if it
-    was taken on the current attention source; else None."""
+    was taken on the current attention code (comments aside); else None."""
     path = os.path.join(ROOT, "profiles", f"attention_{w.name}.md")
     src = os.path.join(ROOT, "paper_2605_06892_gb300", "csrc", "hsa_attention.cu")
     try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        digest = code_digest(open(src).read())
         fields = {}
         for line in open(path):
-            if line.startswith("traffic_per_launch_bytes:") or line.startswith("source_sha256:"):
+            if line.startswith("traffic_per_launch_bytes:") or line.startswith("code_sha256:"):
                 k, v = line.split(":", 1)
                 fields[k.strip()] = v.strip()
-        if fields.get("source_sha256") == sha:
+        if fields.get("code_sha256") == digest:
             return float(fields["traffic_per_launch_bytes"])
     except (OSError, KeyError, ValueError):
         pass

@@ -8,9 +8,12 @@
 // group, which is active at every iteration and so needs no cache.  Warp roles:
 //   warp 0      TMA producer: K and V tiles of the head, 128-byte swizzled,
 //               into a ring of shared-memory slots (rows >= N are zero-filled).
-//   warp 1      tensor-core issuer (one thread): S_t = Q_t K^T into TMEM and
-//               O_t += P_t V from TMEM P and shared V, tcgen05.mma kind::f16.
-//   warps 2-3   idle (they complete the first warpgroup).
+//   warp 1      tensor-core issuer (lane 0 issues, the warp walks the
+//               schedule): S_t = Q_t K^T into TMEM and O_t += P_t V from TMEM
+//               P and shared V, tcgen05.mma kind::f16.
+//   warp 2      K/V watcher: waits for each K/V tile to land, hands it to the
+//               issuer, and gives ring slots back to the producer.
+//   warp 3      idle (it completes the first warpgroup).
 //   warps 4-7   softmax of Q tile 0, warps 8-11 softmax of Q tile 1: each
 //               thread owns one query row (its TMEM lane; a warp may only
 //               reach the lane quarter warp%4), reads its S row,
@@ -18,11 +21,14 @@
 //               the S columns, and at the end normalises O and stores it.
 //   all warps   load the 256 query rows once, by index, into swizzled smem.
 // The two Q tiles ping-pong: while one softmax group works on its scores the
-// tensor core runs the other tile's MMAs.  After the first key tile the
-// probabilities are formed against the running reference maximum without
-// computing the tile's maximum; only if a row sum would pass 2^32 is the tile
-// redone with its exact maximum (and O rescaled in TMEM).  The final division
-// by the running sum makes the result exact whatever reference was used.
+// tensor core runs the other tile's MMAs.  The issuer waits only on hardware
+// named barriers (P of a tile; a K/V tile landed), where the other roles meet
+// it; an mbarrier test on its path would idle the tensor core.  After the
+// first key tile the probabilities are formed against the running reference
+// maximum without computing the tile's maximum; only if a row sum would pass
+// 2^32 is the tile redone with its exact maximum (and O rescaled in TMEM).
+// The final division by the running sum makes the result exact whatever
+// reference was used.
 // Registers: the block launches at 168 per thread; the first warpgroup then
 // gives registers back (setmaxnreg.dec to 96) and the two softmax warpgroups
 // take them (setmaxnreg.inc to 200): 128*96 + 256*200 <= 384*168.
