@@ -486,25 +486,43 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   }
 
   // ---- query rows, by index, into the two swizzled Q tiles (all threads)
+  // Each thread first reads the indices of all its rows, then issues all its
+  // 16-byte loads, then stores them: two dependent round trips to memory in
+  // all rather than two per vector.
   {
     constexpr int kVecPerRow = D / 8;                        // 16-byte vectors per row
+    constexpr int kVecs = kBM * kQT * kVecPerRow;
+    constexpr int kPer = (kVecs + kTcThreads - 1) / kTcThreads;
     const size_t row_stride = (size_t)a.H * D;
-    for (int i = threadIdx.x; i < kBM * kQT * kVecPerRow; i += kTcThreads) {
-      const int row = i / kVecPerRow, c = i % kVecPerRow;
-      const int grow = row0 + row;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (grow < a.n_active) {
-        const int src = a.q_idx ? __ldg(a.q_idx + grow) : grow;
-        if (src >= 0 && src < a.q_rows)
-          v = __ldg(reinterpret_cast<const uint4 *>(a.q + (size_t)src * row_stride +
-                                                    (size_t)h * D) + c);
-        else if (c == 0)
-          set_error(a.err, kErrIndex);
+    int src[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = threadIdx.x + u * kTcThreads;
+      const int grow = row0 + i / kVecPerRow;
+      src[u] = -1;
+      if (i < kVecs && grow < a.n_active) src[u] = a.q_idx ? __ldg(a.q_idx + grow) : grow;
+    }
+    uint4 v[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = threadIdx.x + u * kTcThreads;
+      v[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (src[u] >= 0 && src[u] < a.q_rows)
+        v[u] = __ldg(reinterpret_cast<const uint4 *>(a.q + (size_t)src[u] * row_stride +
+                                                     (size_t)h * D) + i % kVecPerRow);
+      else if (i < kVecs && row0 + i / kVecPerRow < a.n_active && i % kVecPerRow == 0)
+        set_error(a.err, kErrIndex);
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = threadIdx.x + u * kTcThreads;
+      if (i < kVecs) {
+        const int row = i / kVecPerRow, c = i % kVecPerRow;
+        const int t = row / kBM, rr = row % kBM;
+        uint8_t *dst = sQ + t * C::kTileBytes + (c >> 3) * (kBM * 128) + rr * 128 +
+                       (((c & 7) ^ (rr & 7)) << 4);
+        *reinterpret_cast<uint4 *>(dst) = v[u];
       }
-      const int t = row / kBM, rr = row % kBM;
-      uint8_t *dst = sQ + t * C::kTileBytes + (c >> 3) * (kBM * 128) + rr * 128 +
-                     (((c & 7) ^ (rr & 7)) << 4);
-      *reinterpret_cast<uint4 *>(dst) = v;
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
