@@ -467,6 +467,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   const int j0 = wk.j0;
   const int nT = wk.j1 - wk.j0;        // key tiles of this CTA (local index j = 0..nT-1)
 
+  // K or V tile L/2 of this unit's key range (L even: K, odd: V) into its
+  // ring slot, completing on bar_full.  Issued by thread 0, the producer.
+  auto load_kv = [&](int L) {
+    const int slot = L % C::kStages;
+    mbar_expect_tx(&bar_full[slot], C::kTileBytes);
+    const int jg = j0 + (L >> 1);                   // global key tile
+    const bool second = jg >= a.tiles1;
+    const CUtensorMap *map = second ? ((L & 1) ? &tm_v2 : &tm_k2) : ((L & 1) ? &tm_v : &tm_k);
+    const int y = (second ? jg - a.tiles1 : jg) * kBN;
+    uint8_t *dst = sKV + slot * C::kTileBytes;
+#pragma unroll
+    for (int c = 0; c < C::kChunks; ++c)
+      tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, y);
+  };
+  const int withheld = a.inject_stall == 1 ? 1 : -1;   // test hook: V of tile 0 never loads
+  const int n_pre = min(C::kStages, 2 * nT);          // loads issued before the Q tile
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&bar_full[s], 1);
@@ -476,6 +492,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     mbar_init(&bar_o, 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // The first ring's worth of K/V tiles load while the CTA loads its query
+    // rows below.
+    for (int L = 0; L < n_pre; ++L)
+      if (L != withheld) load_kv(L);
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -540,22 +561,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     if (warp == 0) {
       // ------------------------------------------------ TMA producer
       if (lane == 0) {
-        int issued = 0;
-        const int withheld = a.inject_stall == 1 ? 1 : -1;   // test hook
-        for (int L = 0; L < 2 * nT; ++L) {
+        int issued = n_pre;
+        for (int L = n_pre; L < 2 * nT; ++L) {
           const int slot = L % C::kStages, use = L / C::kStages;
           if (use > 0 && !mbar_wait(&bar_empty[slot], (use - 1) & 1, &abort_flag, a.err)) break;
           if (L == withheld) continue;
-          mbar_expect_tx(&bar_full[slot], C::kTileBytes);
-          const int jg = j0 + (L >> 1);                   // global key tile
-          const bool second = jg >= a.tiles1;
-          const CUtensorMap *map = second ? ((L & 1) ? &tm_v2 : &tm_k2)
-                                          : ((L & 1) ? &tm_v : &tm_k);
-          const int y = (second ? jg - a.tiles1 : jg) * kBN;
-          uint8_t *dst = sKV + slot * C::kTileBytes;
-#pragma unroll
-          for (int c = 0; c < C::kChunks; ++c)
-            tma_load_2d(dst + c * (kBN * 128), map, &bar_full[slot], h * D + c * 64, y);
+          load_kv(L);
           issued = L + 1;
         }
         // Drain: every issued copy has landed before the CTA may exit.  A
