@@ -175,6 +175,55 @@ radix_scatter_kernel(const uint32_t *__restrict__ kin, const int32_t *__restrict
   }
 }
 
+// ------------------------------------------------ small layers: rank by count
+//
+// For N <= kRankMaxN every block holds all N keys in shared memory, and a
+// token's rank is the number of tokens ordered before it by (key, index):
+// exactly the ranks of the stable sort, in one launch instead of fourteen.
+// A block takes 32 tokens (its lanes) and splits the key range over its 8
+// warps; the partial counts are summed in shared memory.  The keys are the
+// same order-preserving transform as radix_key_kernel's.
+constexpr int kRankMaxN = 12288;                        // keys fill <= 48 KB
+constexpr int kRankThreads = 256;
+constexpr int kRankTokens = 32;
+
+__global__ void __launch_bounds__(kRankThreads)
+rank_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStarts gs,
+                      int32_t *__restrict__ group_of, unsigned *err) {
+  extern __shared__ uint32_t skey[];
+  __shared__ int part[kRankThreads / 32][kRankTokens];
+  for (int m = threadIdx.x; m < N; m += kRankThreads) {
+    const float f = stat[m];
+    uint32_t u = __float_as_uint(f);
+    if (blockIdx.x == 0 && !isfinite(f)) set_error(err, kErrNonfinite);
+    if (u == 0x80000000u) u = 0u;                          // -0 ranks with +0
+    skey[m] = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // float order as uint order
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int n = blockIdx.x * kRankTokens + lane;
+  const uint32_t kn = n < N ? skey[n] : 0u;
+  const int per = (N + kRankThreads / 32 - 1) / (kRankThreads / 32);
+  const int m0 = w * per, m1 = min(N, m0 + per);
+  int r = 0;
+#pragma unroll 4
+  for (int m = m0; m < m1; ++m) {
+    const uint32_t km = skey[m];                           // the same word for every lane
+    r += (km < kn) + ((km == kn) & (m < n));
+  }
+  part[w][lane] = r;
+  __syncthreads();
+  if (w == 0 && n < N) {
+    int rank = 0;
+#pragma unroll
+    for (int i = 0; i < kRankThreads / 32; ++i) rank += part[i][lane];
+    int g = 0;
+    for (int k = 0; k < K; ++k)
+      if (rank >= gs.start[k] && rank < gs.start[k] + gs.count[k]) g = k;
+    group_of[n] = g;
+  }
+}
+
 __global__ void __launch_bounds__(kSortThreads)
 group_assign_kernel(const int32_t *__restrict__ sorted_tokens, int N, int K, GroupStarts gs,
               int32_t *__restrict__ group_of) {
@@ -283,6 +332,19 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
   cudaStream_t s = (cudaStream_t)stream;
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
+  GroupStarts gs{};
+  int r = 0;
+  for (int k = K - 1; k >= 0; --k) {
+    gs.start[k] = r;
+    gs.count[k] = counts[k];
+    r += counts[k];
+  }
+  if (N <= kRankMaxN) {
+    count_launches(1);
+    rank_partition_kernel<<<(N + kRankTokens - 1) / kRankTokens, kRankThreads,
+                            (size_t)N * sizeof(uint32_t), s>>>(stat, N, K, gs, group_of, err);
+    return launch_status();
+  }
   const int ew_blocks = (int)std::min<long long>((N + kSortThreads - 1) / kSortThreads,
                                                  (long long)sm_count() * 8);
   count_launches(1);
@@ -296,13 +358,6 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
     count_launches(1);
     radix_scatter_kernel<<<L.tiles, kSortThreads, 0, s>>>(keys[in], vals[in], keys[out], vals[out], N,
                                                      8 * pass, hist, L.tiles);
-  }
-  GroupStarts gs{};
-  int r = 0;
-  for (int k = K - 1; k >= 0; --k) {
-    gs.start[k] = r;
-    gs.count[k] = counts[k];
-    r += counts[k];
   }
   count_launches(1);
   group_assign_kernel<<<ew_blocks, kSortThreads, 0, s>>>(vals[0], N, K, gs, group_of);
