@@ -20,7 +20,6 @@ not available, so these tensors stand in for them with the paper's shapes):
 """
 from __future__ import annotations
 
-import math
 from dataclasses import dataclass, field
 
 import torch

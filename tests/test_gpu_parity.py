@@ -7,7 +7,6 @@ the condition |x| + |v dsigma|; bf16 attention within max |err| <= 2e-2 and
 relative L2 error <= 1e-2 of the fp64 oracle fed the same bf16 inputs; fp32
 attention within 1e-4.
 """
-import math
 
 import pytest
 import torch
