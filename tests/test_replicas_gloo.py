@@ -31,7 +31,7 @@ def _worker(rank, world, port, times, out):
 def test_max_over_ranks_gloo():
     world = 2
     times = [3.5, 7.25]
-    out = mp.Manager().dict()
+    out = mp.get_context("spawn").Manager().dict()
     mp.spawn(_worker, args=(world, _free_port(), times, out), nprocs=world, join=True)
     assert out[0] == out[1] == max(times)
 
