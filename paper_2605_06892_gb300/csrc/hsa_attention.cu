@@ -825,8 +825,10 @@ attn_combine_kernel(const float *__restrict__ ws_o, const float *__restrict__ ws
 
 constexpr int kF32Threads = 128;
 constexpr int kF32Keys = 32;
+constexpr int kF32Dims = 8;      // dimensions per thread
 
-// TPQ = D/32 threads cooperate on one query; thread slice s owns dimensions
+// TPQ = D/8 threads cooperate on one query (8 dimensions each, so that small
+// layers still give the GPU enough threads); thread slice s owns dimensions
 // s, s+TPQ, s+2*TPQ, ... so that the slices of one query hit distinct banks.
 template <int D>
 __global__ void __launch_bounds__(kF32Threads)
@@ -835,7 +837,7 @@ attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
                 const float *__restrict__ kb, const float *__restrict__ vb,
                 float *__restrict__ out, int n_active, int N, int H, int q_rows, float scale,
                 unsigned *err) {
-  constexpr int TPQ = D / 32;
+  constexpr int TPQ = D / kF32Dims;
   constexpr int QPB = kF32Threads / TPQ;
   __shared__ float sK[kF32Keys][D];
   __shared__ float sV[kF32Keys][D];
@@ -843,21 +845,21 @@ attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
   const int ql = threadIdx.x / TPQ, sl = threadIdx.x % TPQ;
   const int j = blockIdx.x * QPB + ql;
   const bool active = j < n_active;
-  float qv[32], o[32];
+  float qv[kF32Dims], o[kF32Dims];
   bool row_ok = false;
   if (active) {
     const int src = q_idx ? q_idx[j] : j;
     row_ok = src >= 0 && src < q_rows;
     if (!row_ok && sl == 0) set_error(err, kErrIndex);
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
+    for (int i = 0; i < kF32Dims; ++i)
       qv[i] = row_ok ? q[((size_t)src * H + h) * D + sl + TPQ * i] : 0.f;
   } else {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) qv[i] = 0.f;
+    for (int i = 0; i < kF32Dims; ++i) qv[i] = 0.f;
   }
 #pragma unroll
-  for (int i = 0; i < 32; ++i) o[i] = 0.f;
+  for (int i = 0; i < kF32Dims; ++i) o[i] = 0.f;
   float m = -INFINITY, l = 0.f;
   for (int n0 = 0; n0 < N; n0 += kF32Keys) {
     __syncthreads();
@@ -881,7 +883,7 @@ attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
     for (int kk = 0; kk < kF32Keys; ++kk) {
       float dot = 0.f;
 #pragma unroll
-      for (int i = 0; i < 32; ++i) dot = fmaf(qv[i], sK[kk][sl + TPQ * i], dot);
+      for (int i = 0; i < kF32Dims; ++i) dot = fmaf(qv[i], sK[kk][sl + TPQ * i], dot);
 #pragma unroll
       for (int o2 = 1; o2 < TPQ; o2 <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o2);
       sc[kk] = (n0 + kk < N) ? dot * scale : -INFINITY;
@@ -891,20 +893,20 @@ attn_f32_kernel(const float *__restrict__ q, const int32_t *__restrict__ q_idx,
     const float corr = expf(m - m_new);
     l *= corr;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) o[i] *= corr;
+    for (int i = 0; i < kF32Dims; ++i) o[i] *= corr;
 #pragma unroll
     for (int kk = 0; kk < kF32Keys; ++kk) {
       const float p = expf(sc[kk] - m_new);
       l += p;
 #pragma unroll
-      for (int i = 0; i < 32; ++i) o[i] = fmaf(p, sV[kk][sl + TPQ * i], o[i]);
+      for (int i = 0; i < kF32Dims; ++i) o[i] = fmaf(p, sV[kk][sl + TPQ * i], o[i]);
     }
     m = m_new;
   }
   if (active) {
     const float inv = 1.f / l;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) out[((size_t)j * H + h) * D + sl + TPQ * i] = o[i] * inv;
+    for (int i = 0; i < kF32Dims; ++i) out[((size_t)j * H + h) * D + sl + TPQ * i] = o[i] * inv;
   }
 }
 
@@ -1050,7 +1052,7 @@ template <int D>
 int launch_f32(const void *q, const int32_t *q_idx, int n_active, const void *k_cache,
                const void *v_cache, int rows1, const void *k_base, const void *v_base, int rows2,
                int H, float scale, void *out, cudaStream_t stream, unsigned *err) {
-  constexpr int QPB = kF32Threads / (D / 32);
+  constexpr int QPB = kF32Threads / (D / kF32Dims);
   const int N = rows1 + rows2;
   const dim3 grid((n_active + QPB - 1) / QPB, H);
   count_launches(1);
