@@ -330,9 +330,7 @@ def run_hsa(args, dist, rank, world, local_rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) Q/K/V, lognormal statistic; no model weights)",
-        "config": {"workload": f"{w.name}: N={w.N} ({w.grid[0]}x{w.grid[1]}x{w.grid[2]}), "
-                               f"H={w.H}, D={w.D}, budgets={list(budgets)}, "
-                               f"counts={list(L.counts)}, T={T}, iterations={L.iters}",
+        "config": {"workload": workload_desc(w, L.counts),
                    "per_iteration": per_iter, "parallelism": f"replicas x{world}",
                    "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
                    "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
@@ -586,6 +584,13 @@ def cpu_baseline(w, L=None, target_s=15.0):
                       f"{t:.1f} s single-threaded"}
 
 
+def workload_desc(w, counts) -> str:
+    """The workload as both arms name it in `config.workload`."""
+    return (f"{w.name}: N={w.N} ({w.grid[0]}x{w.grid[1]}x{w.grid[2]}), H={w.H}, D={w.D}, "
+            f"budgets={list(w.budgets)}, counts={list(counts)}, T={w.T}, "
+            f"iterations={list(w.iters)}")
+
+
 def run_reference(args, dist, rank, world):
     """The oracle as the reference arm: each step is a bounded sample of the
     workload (4 query rows per iteration), timed on the host cores."""
@@ -610,7 +615,7 @@ def run_reference(args, dist, rank, world):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * tot_t / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": f"{w.name}: N={w.N}, H={w.H}, D={w.D}"},
+        "config": {"workload": workload_desc(w, counts)},
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
