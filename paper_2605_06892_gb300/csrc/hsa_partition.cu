@@ -380,11 +380,11 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
     const bool full = iter < m || iter > T - m - 1;
     if (full || iter % (T / budgets[k]) == 0) mask |= 1u << k;
   }
-  // Chunks of at least 4096 tokens, at most one block per SM.
+  // Chunks of whole 1024-token rounds, at most one block per SM: a layer of
+  // up to 152 * 1024 tokens is compacted in one round per block.
   const int sms = sm_count();
   long long chunk = ((long long)N + sms - 1) / sms;
   chunk = ((chunk + kActThreads - 1) / kActThreads) * kActThreads;
-  if (chunk < 4096) chunk = 4096;
   const int blocks = (int)(((long long)N + chunk - 1) / chunk);
   cudaStream_t s = (cudaStream_t)stream;
   unsigned *err = device_error_word();
