@@ -281,15 +281,17 @@ static_assert(128 * kRegsLow + 256 * kRegsHigh <= kTcThreads * kLaunchRegs,
               "register split exceeds the launch allocation");
 constexpr int kTmemCols = 512;
 // Named barriers (hardware, not in shared memory): 1 = teardown of the whole
-// CTA; kBarP0 + t = P of Q tile t is in TMEM (its 128 softmax threads and the
-// issuing warp meet); kBarKV0 + s = the K/V tile in ring slot s has landed
-// (the K/V watcher warp and the issuing warp meet).  Every party syncs
-// (a rendezvous, never a lone arrive) once per hand-off in the same order, so
-// no party can run a whole round ahead and the barrier instances always pair
-// up, also after a failed wait.
+// CTA; kBarK0 = the first K tile has landed (the K/V watcher and the issuing
+// warp meet once); kBarP0 + t = P of Q tile t is in TMEM, for key tile j (its
+// 128 softmax threads, the issuing warp and the K/V watcher meet; at the
+// meeting for P_0(j) the watcher has seen V_j and K_(j+1) land).  Every party
+// syncs (a rendezvous, never a lone arrive) once per hand-off in the same
+// order, so no party can run a whole round ahead and the barrier instances
+// always pair up, also after a failed wait.
 constexpr int kBarTeardown = 1;
 constexpr int kBarP0 = 2;
-constexpr int kBarKV0 = 4;
+constexpr int kBarK0 = 4;
+constexpr int kMeetP = kBM + 64;   // threads at a P meeting
 
 template <int D>
 struct TcCfg {
@@ -555,7 +557,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   // The warpgroups' code paths never rejoin below: each ends with its own
   // teardown on named barrier 1, so each path is compiled for its own
   // register budget.
-  static_assert(kBarKV0 + C::kStages <= 16, "named barrier ids");
+
   if (warp < 4) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
     if (warp == 0) {
@@ -586,11 +588,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       // mbarrier test on this path costs about a hundred clocks while an S
       // group's operand reads fill the shared-memory bandwidth; a named
       // barrier whose other parties have already arrived costs far less.
-      // So the issuer waits on named barriers only: kBarKV0 + slot (the K/V
-      // watcher saw the tile land) and kBarP0 + t (the softmax of Q tile t
-      // stored P).  Every party meets it exactly once per hand-off whatever
-      // happens, so each sync completes; after an abort the warp keeps its
-      // syncs but issues nothing more.
+      // So the issuer waits on named barriers only, two per key tile:
+      // kBarP0 + t, where the softmax of Q tile t has stored P and the K/V
+      // watcher has seen the tiles the next MMAs read land (once, before the
+      // loop, kBarK0 for the first K tile).  Every party meets it exactly once
+      // per hand-off whatever happens, so each sync completes; after an abort
+      // the warp keeps its syncs but issues nothing more.
       const bool leader = lane == 0;
       constexpr uint32_t kIdS = idesc_bf16(kBM, kBN, 0);
       constexpr uint32_t kIdO = idesc_bf16(kBM, D, 1);
@@ -621,15 +624,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         for (int k = 0; k < kBN / 16; ++k)
           mma_ts(to, tp + 8 * k, dv + ((k * 2048) >> 4), kIdO, (acc || k > 0) ? 1u : 0u);
       };
-      auto kv_ready = [&](int L) {
-        named_barrier_sync(kBarKV0 + L % C::kStages, 64);
-        fence_after();
-      };
       auto p_ready = [&](int t) {
-        named_barrier_sync(kBarP0 + t, kBM + 32);
+        named_barrier_sync(kBarP0 + t, kMeetP);
         fence_after();
       };
-      kv_ready(0);
+      named_barrier_sync(kBarK0, 64);               // K_0 has landed
+      fence_after();
       if (leader && !abort_flag) {
         issue_s(0, 0);
         mma_commit(&bar_s[0]);
@@ -639,13 +639,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       for (int j = 0; j < nT; ++j) {
         const int Lv = 2 * j + 1, Lk = 2 * j + 2;
         const bool more = j + 1 < nT;
-        kv_ready(Lv);
-        p_ready(0);
+        p_ready(0);                                 // P_0(j); V_j and K_(j+1) landed
         const bool go = leader && !abort_flag;
-        if (go) issue_o(0, Lv, j > 0);
-        if (more) {
-          kv_ready(Lk);
-          if (go) {
+        if (go) {
+          issue_o(0, Lv, j > 0);
+          if (more) {
             issue_s(0, Lk);
             mma_commit(&bar_s[0]);
           }
@@ -668,34 +666,41 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       __syncwarp();
     } else if (warp == 2) {
       // ------------------------------------------------ K/V watcher
-      // Waits (bounded) for each K/V tile to land and meets the issuer on
-      // the slot's named barrier.  It meets it once per tile even after a
-      // failed wait, so the issuer never waits forever.  It also gives slots
-      // back to the producer, so the issuer commits nothing for them: once
-      // S_1 of key tile j has completed (the tensor core runs its MMAs in
-      // order), K_j and V_(j-1) have been read by every MMA that uses them.
-      // It waits for that right after meeting the issuer for V_j: S_1 of key
-      // tile j+1 needs K_(j+1), which it has not handed over yet, so the
-      // phase it waits for is never overtaken.  After a failure it gives
-      // nothing back, so no slot is refilled while a copy into it may still
-      // be in flight.
+      // Waits (bounded) for the K/V tiles to land and hands them to the
+      // issuer at the P meetings: V_j and K_(j+1) before P_0(j) (K_0 alone,
+      // before the loop).  It also gives ring slots back to the producer, so
+      // the issuer commits nothing for them: once S_1 of key tile j has
+      // completed (the tensor core runs its MMAs in order), K_j and V_(j-1)
+      // have been read by every MMA that uses them.  It waits for that between
+      // the meetings for P_0(j) and P_1(j); S_1 of key tile j+1 is issued only
+      // after the meeting for P_1(j), so the phase it waits for is never
+      // overtaken.  It meets the issuer at every meeting even after a failed
+      // wait, so the issuer never waits forever, and after a failure it gives
+      // nothing back, so no slot is refilled while a copy into it may still be
+      // in flight.
       bool live = true;
-      auto give_back = [&](int L) {
-        if (lane == 0) mbar_arrive(&bar_empty[L % C::kStages]);
-      };
-      for (int L = 0; L < 2 * nT; ++L) {
+      auto landed = [&](int L) {
         if (live)
           live = __all_sync(0xffffffffu, mbar_wait(&bar_full[L % C::kStages],
                                                    (L / C::kStages) & 1, &abort_flag, a.err));
-        named_barrier_sync(kBarKV0 + L % C::kStages, 64);
-        if ((L & 1) && live) {                     // L = V_j, j = L / 2
-          const int j = L >> 1;
+      };
+      auto give_back = [&](int L) {
+        if (lane == 0) mbar_arrive(&bar_empty[L % C::kStages]);
+      };
+      landed(0);
+      named_barrier_sync(kBarK0, 64);
+      for (int j = 0; j < nT; ++j) {
+        landed(2 * j + 1);                         // V_j
+        if (j + 1 < nT) landed(2 * j + 2);         // K_(j+1)
+        named_barrier_sync(kBarP0, kMeetP);
+        if (live) {
           live = __all_sync(0xffffffffu, mbar_wait(&bar_s[1], j & 1, &abort_flag, a.err));
           if (live) {
             give_back(2 * j);                      // K_j
             if (j > 0) give_back(2 * j - 1);       // V_(j-1)
           }
         }
+        named_barrier_sync(kBarP0 + 1, kMeetP);
       }
     }
     fence_before();
@@ -736,7 +741,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         tmem_wait_st();
       }
       fence_before();
-      named_barrier_sync(kBarP0 + t, kBM + 32);
+      named_barrier_sync(kBarP0 + t, kMeetP);
     }
     if (ok && wk.piece >= 0 && mbar_wait(&bar_o, 0, &abort_flag, a.err)) {
       // Piece of a split unit: unnormalised O, maximum and sum, for the combine.
