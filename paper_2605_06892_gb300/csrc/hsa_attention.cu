@@ -11,8 +11,9 @@
 //   warp 1      tensor-core issuer (lane 0 issues, the warp walks the
 //               schedule): S_t = Q_t K^T into TMEM and O_t += P_t V from TMEM
 //               P and shared V, tcgen05.mma kind::f16.
-//   warp 2      K/V watcher: waits for each K/V tile to land, hands it to the
-//               issuer, and gives ring slots back to the producer.
+//   warp 2      K/V watcher: waits for the K/V tiles to land, hands them to
+//               the issuer at the P meetings, and gives ring slots back to
+//               the producer.
 //   warp 3      idle (it completes the first warpgroup).
 //   warps 4-7   softmax of Q tile 0, warps 8-11 softmax of Q tile 1: each
 //               thread owns one query row (its TMEM lane; a warp may only
@@ -22,8 +23,9 @@
 //   all warps   load the 256 query rows once, by index, into swizzled smem.
 // The two Q tiles ping-pong: while one softmax group works on its scores the
 // tensor core runs the other tile's MMAs.  The issuer waits only on hardware
-// named barriers (P of a tile; a K/V tile landed), where the other roles meet
-// it; an mbarrier test on its path would idle the tensor core.  After the
+// named barriers, two per key tile (P of a tile, with the K/V tiles the next
+// MMAs read), where the other roles meet it; an mbarrier test on its path
+// would idle the tensor core.  After the
 // first key tile the probabilities are formed against the running reference
 // maximum without computing the tile's maximum; only if a row sum would pass
 // 2^32 is the tile redone with its exact maximum (and O rescaled in TMEM).
