@@ -183,9 +183,13 @@ radix_scatter_kernel(const uint32_t *__restrict__ kin, const int32_t *__restrict
 // A block takes 32 tokens (its lanes) and splits the key range over its 8
 // warps; the partial counts are summed in shared memory.  The keys are the
 // same order-preserving transform as radix_key_kernel's.
-constexpr int kRankMaxN = 12288;                        // keys fill <= 48 KB
 constexpr int kRankThreads = 256;
 constexpr int kRankTokens = 32;
+// The keys (dynamic) and the partial counts (static) stay within the 48 KB a
+// block gets without opting in to more shared memory.
+constexpr int kRankMaxN = (48 * 1024 - (kRankThreads / 32) * kRankTokens * 4) / 4;   // 12032
+static_assert(kRankMaxN * 4 + (kRankThreads / 32) * kRankTokens * 4 <= 48 * 1024,
+              "rank partition shared memory");
 
 __global__ void __launch_bounds__(kRankThreads)
 rank_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStarts gs,
@@ -221,6 +225,210 @@ rank_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStarts 
     for (int k = 0; k < K; ++k)
       if (rank >= gs.start[k] && rank < gs.start[k] + gs.count[k]) g = k;
     group_of[n] = g;
+  }
+}
+
+// ------------------------------------------------ mid-size layers: select
+//
+// A token's group depends only on which group boundaries its rank passes:
+// rank >= start[k] for k = 0 .. K-2 (group K-1 holds the lowest ranks), and
+// rank >= b holds exactly when (key, token) >= the pair of rank b in the
+// (key, token) order.  So for kRankMaxN < N <= kSelectMaxN one block loads the
+// N keys into shared memory, finds the pair of each boundary rank (a radix
+// select: four 8-bit digit passes, each a histogram of the keys that share
+// the boundary's digits so far, then the boundary's position among the keys
+// equal to its key, counted in token order) and compares every token with
+// those pairs.  One launch instead of fourteen, and the same ranks as the
+// stable sort.
+constexpr int kSelectThreads = 1024;
+constexpr int kSelectMaxN = 49152;                     // keys: 192 KB of shared memory
+constexpr int kMaxBounds = kMaxGroups - 1;
+
+__device__ __forceinline__ uint32_t order_key(float f) {
+  uint32_t u = __float_as_uint(f);
+  if (u == 0x80000000u) u = 0u;                          // -0 ranks with +0
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);     // float order as uint order
+}
+
+__global__ void __launch_bounds__(kSelectThreads)
+select_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStarts gs,
+                        int32_t *__restrict__ group_of, unsigned *err) {
+  extern __shared__ uint4 skey4[];                      // the N keys, padded to whole uint4
+  uint32_t *skey = reinterpret_cast<uint32_t *>(skey4);
+  __shared__ uint32_t hist[kMaxBounds][256];
+  __shared__ uint32_t pre[kMaxBounds];      // boundary key digits found so far
+  __shared__ int below[kMaxBounds];         // keys ordered below that digit prefix
+  __shared__ int slot[kMaxBounds];          // histogram of the boundary's prefix
+  __shared__ uint32_t dpre[kMaxBounds];     // distinct prefixes, ascending
+  __shared__ int nd;
+  __shared__ unsigned long long thr[kMaxBounds];   // boundary pair (key << 32 | token)
+  __shared__ int warp_tot[kSelectThreads / 32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int nb = K - 1;
+  const int n4 = (N + 3) >> 2;
+  // boundary j is searched when 0 < start[j] < N (rank 0 is passed by every
+  // token, rank N by none)
+  auto searched = [&](int j) { return gs.start[j] > 0 && gs.start[j] < N; };
+  if ((reinterpret_cast<uintptr_t>(stat) & 15) == 0) {
+    for (int i = threadIdx.x; i < n4; i += kSelectThreads) {
+      float4 f;
+      if (4 * i + 3 < N) {
+        f = reinterpret_cast<const float4 *>(stat)[i];
+      } else {
+        f.x = stat[4 * i];
+        f.y = 4 * i + 1 < N ? stat[4 * i + 1] : 0.f;
+        f.z = 4 * i + 2 < N ? stat[4 * i + 2] : 0.f;
+        f.w = 0.f;
+      }
+      if (!(isfinite(f.x) && isfinite(f.y) && isfinite(f.z) && isfinite(f.w)))
+        set_error(err, kErrNonfinite);
+      skey4[i] = make_uint4(order_key(f.x), order_key(f.y), order_key(f.z), order_key(f.w));
+    }
+  } else {
+    for (int n = threadIdx.x; n < 4 * n4; n += kSelectThreads) {
+      const float f = n < N ? stat[n] : 0.f;
+      if (!isfinite(f)) set_error(err, kErrNonfinite);
+      skey[n] = order_key(f);
+    }
+  }
+  if (threadIdx.x == 0) {
+    nd = 1;
+    dpre[0] = 0u;
+  }
+  if (threadIdx.x < kMaxBounds) {
+    pre[threadIdx.x] = 0u;
+    below[threadIdx.x] = 0;
+    slot[threadIdx.x] = 0;
+  }
+  __syncthreads();
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    const int n_hist = nd;
+    for (int i = threadIdx.x; i < n_hist * 256; i += kSelectThreads) hist[i >> 8][i & 255] = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < n4; i += kSelectThreads) {
+      const uint4 k4 = skey4[i];
+      const uint32_t kk[4] = {k4.x, k4.y, k4.z, k4.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (4 * i + e >= N) break;                     // padding
+        const uint32_t key = kk[e];
+        const uint32_t hi = pass == 0 ? 0u : key >> (shift + 8);
+        for (int q = 0; q < n_hist; ++q) {             // few distinct prefixes
+          const uint32_t v = dpre[q];
+          if (v >= hi) {
+            if (v == hi) atomicAdd(&hist[q][(key >> shift) & 255u], 1u);
+            break;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    // warp j picks boundary j's digit: the bin where its rank falls
+    if (w < nb && searched(w)) {
+      const int target = gs.start[w] - below[w];       // rank among the prefix's keys
+      const uint32_t *h = hist[slot[w]];
+      int c[8], sum = 0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { c[i] = (int)h[8 * lane + i]; sum += c[i]; }
+      int incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      const int excl = incl - sum;
+      if (target >= excl && target < incl) {           // exactly one lane
+        int cum = excl, d = 8 * lane;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (target < cum + c[i]) { d = 8 * lane + i; break; }
+          cum += c[i];
+        }
+        pre[w] = (pre[w] << 8) | (uint32_t)d;
+        below[w] += cum;                               // keys below the longer prefix
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {                            // distinct prefixes, ascending
+      int m = 0;
+      for (int j = 0; j < nb; ++j) {
+        if (!searched(j)) continue;
+        const uint32_t v = pre[j];
+        int pos = 0;
+        while (pos < m && dpre[pos] < v) ++pos;
+        if (pos == m || dpre[pos] != v) {
+          for (int q = m; q > pos; --q) dpre[q] = dpre[q - 1];
+          dpre[pos] = v;
+          ++m;
+        }
+      }
+      for (int j = 0; j < nb; ++j) {
+        if (!searched(j)) continue;
+        int pos = 0;
+        while (dpre[pos] != pre[j]) ++pos;
+        slot[j] = pos;
+      }
+      nd = m > 0 ? m : 1;
+    }
+    __syncthreads();
+  }
+  // Boundary j's pair: its key pre[j] and the token of rank start[j] - below[j]
+  // among the tokens with that key in token order.  Thread t counts a
+  // contiguous run of tokens; an odd run length keeps the threads of a warp
+  // on different shared-memory banks.
+  const int run = ((N + kSelectThreads - 1) / kSelectThreads) | 1;
+  const int r0 = min(N, threadIdx.x * run), r1 = min(N, r0 + run);
+  for (int j = 0; j < nb; ++j) {
+    const int b = gs.start[j];
+    if (!searched(j)) {                                // the same for every thread
+      if (threadIdx.x == 0) thr[j] = b <= 0 ? 0ull : ~0ull;
+      continue;
+    }
+    const uint32_t kj = pre[j];
+    int eq = 0;
+    for (int n = r0; n < r1; ++n) eq += skey[n] == kj;
+    // exclusive block sum of eq
+    int incl = eq;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) warp_tot[w] = incl;
+    __syncthreads();
+    if (w == 0) {
+      const int x = warp_tot[lane];
+      int inc = x;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += t;
+      }
+      warp_tot[lane] = inc - x;
+    }
+    __syncthreads();
+    const int before = warp_tot[w] + incl - eq;
+    const int need = b - below[j];
+    if (need >= before && need < before + eq) {
+      int seen = before;
+      for (int n = r0; n < r1; ++n) {
+        if (skey[n] != kj) continue;
+        if (seen == need) {
+          thr[j] = ((unsigned long long)kj << 32) | (unsigned)n;
+          break;
+        }
+        ++seen;
+      }
+    }
+    __syncthreads();                                   // warp_tot is reused
+  }
+  __syncthreads();
+  for (int n = threadIdx.x; n < N; n += kSelectThreads) {
+    const unsigned long long kn = ((unsigned long long)skey[n] << 32) | (unsigned)n;
+    int passed = 0;
+    for (int j = 0; j < nb; ++j) passed += kn >= thr[j];
+    group_of[n] = K - 1 - passed;
   }
 }
 
@@ -343,6 +551,21 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
     count_launches(1);
     rank_partition_kernel<<<(N + kRankTokens - 1) / kRankTokens, kRankThreads,
                             (size_t)N * sizeof(uint32_t), s>>>(stat, N, K, gs, group_of, err);
+    return launch_status();
+  }
+  if (N <= kSelectMaxN) {
+    static std::atomic<int> configured[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return HSA_ERR_CUDA;
+    if (!configured[dev].load()) {
+      if (cudaFuncSetAttribute(select_partition_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kSelectMaxN * (int)sizeof(uint32_t)) != cudaSuccess)
+        return HSA_ERR_CUDA;
+      configured[dev].store(1);
+    }
+    count_launches(1);
+    select_partition_kernel<<<1, kSelectThreads, (size_t)((N + 3) / 4) * sizeof(uint4), s>>>(
+        stat, N, K, gs, group_of, err);
     return launch_status();
   }
   const int ew_blocks = (int)std::min<long long>((N + kSortThreads - 1) / kSortThreads,

@@ -1,8 +1,9 @@
 """The library's launch counter (hsa_launch_count) on the GPU: each entry point
 adds the number of kernels it enqueues, which is what the bench reports as its
-launch count.  Partition of a layer of at most 12288 tokens is one ranking
-launch; larger layers take the 4-pass radix sort (key, then histogram + scan +
-scatter per pass) plus the group assignment.  bf16 attention with a workspace
+launch count.  Partition of a layer of at most 49152 tokens is one launch (a
+ranking up to 12032 tokens, then a one-block boundary select); larger layers
+take the 4-pass radix sort (key, then histogram + scan + scatter per pass) plus
+the group assignment.  bf16 attention with a workspace
 adds a combine launch exactly when its last wave is split along the keys."""
 import pytest
 import torch
@@ -36,14 +37,16 @@ def test_launch_counts(hsa):
     stat = synth.lognormal_stat(N, 1.0, 3).to(DEV)
     g = torch.empty(N, dtype=torch.int32, device=DEV)
     ws = torch.empty(hsa.hsa_partition_workspace_bytes(N), dtype=torch.uint8, device=DEV)
-    # a layer this small is ranked in one launch; a large one takes the radix sort
+    # up to 49152 tokens the partition takes one launch (rank by count, then
+    # boundary select); beyond, the radix sort takes fourteen
     assert _delta(hsa, lambda: hsa.hsa_partition(stat, T, budgets, counts, g, ws)) == 1
-    Nb = 20000
-    stat_b = synth.lognormal_stat(Nb, 1.0, 4).to(DEV)
-    g_b = torch.empty(Nb, dtype=torch.int32, device=DEV)
-    ws_b = torch.empty(hsa.hsa_partition_workspace_bytes(Nb), dtype=torch.uint8, device=DEV)
-    assert _delta(hsa, lambda: hsa.hsa_partition(stat_b, T, budgets, (5000, 15000), g_b,
-                                                 ws_b)) == 14
+    for Nb, launches in ((20000, 1), (300000, 14)):
+        stat_b = synth.lognormal_stat(Nb, 1.0, 4).to(DEV)
+        g_b = torch.empty(Nb, dtype=torch.int32, device=DEV)
+        ws_b = torch.empty(hsa.hsa_partition_workspace_bytes(Nb), dtype=torch.uint8, device=DEV)
+        assert _delta(hsa, lambda: hsa.hsa_partition(stat_b, T, budgets,
+                                                     (Nb // 4, Nb - Nb // 4), g_b,
+                                                     ws_b)) == launches
     idx = torch.empty(N, dtype=torch.int32, device=DEV)
     pos = torch.empty(N, dtype=torch.int32, device=DEV)
     assert _delta(hsa, lambda: hsa.hsa_partition_active(g, T, budgets, 0, idx, pos)) == 1

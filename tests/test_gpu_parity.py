@@ -81,6 +81,31 @@ def test_partition_ties_signed_zero_ragged(hsa, N):
     _no_device_error(hsa)
 
 
+@pytest.mark.parametrize("N", [12032, 12033, 20000, 49152, 49153, 300001])
+def test_partition_paths_many_and_empty_groups(hsa, N):
+    """Each of the three partition paths (rank by count up to 12032 tokens, one
+    block selecting the group boundaries up to 49152, the radix sort beyond)
+    against the oracle: 1 to 32 groups with random cuts, a run of equal values
+    straddling boundaries, and empty groups at either end."""
+    g = torch.Generator().manual_seed(N)
+    stat = synth.lognormal_stat(N, 1.0, 11)
+    stat[N // 3: N // 3 + 3000] = stat[7]             # ties across several boundaries
+    stat[5] = -0.0
+    stat[6] = 0.0
+    for K in (1, 2, 5, 32):
+        budgets = (40,) * K
+        cut = sorted(torch.randint(0, N + 1, (K - 1,), generator=g).tolist())
+        b = [0] + cut + [N]
+        counts = tuple(b[k + 1] - b[k] for k in range(K))
+        assert torch.equal(_gpu_partition(hsa, stat, 40, budgets, counts),
+                           oracle.partition(stat, 40, budgets, counts)), (K, counts)
+    lo = int((stat < stat[7]).sum())                  # a cut inside the run of ties
+    for counts in ((0, N, 0), (N, 0, 0), (0, 0, N), (N - lo - 1000, 1000, lo)):
+        assert torch.equal(_gpu_partition(hsa, stat, 40, (40, 20, 10), counts),
+                           oracle.partition(stat, 40, (40, 20, 10), counts)), counts
+    _no_device_error(hsa)
+
+
 def test_partition_single_group_and_empty_groups(hsa):
     stat = synth.lognormal_stat(5000, 1.0, 3)
     for budgets, counts in (((8,), (5000,)), ((8, 4, 2), (0, 5000, 0)), ((8, 1), (4999, 1))):
@@ -107,6 +132,13 @@ def test_partition_errors(hsa):
     bad[17] = float("-inf")
     hsa.hsa_partition(bad, 40, (40, 10), (50, 50), g, ws)
     assert hsa.hsa_get_device_error() == -5
+    for n_big in (20000, 300000):                     # the select and radix paths
+        big = torch.rand(n_big).to(DEV)
+        big[n_big - 3] = float("nan")
+        gb = torch.empty(n_big, dtype=torch.int32, device=DEV)
+        wsb = torch.empty(hsa.hsa_partition_workspace_bytes(n_big), dtype=torch.uint8, device=DEV)
+        hsa.hsa_partition(big, 40, (40, 10), (n_big // 2, n_big - n_big // 2), gb, wsb)
+        assert hsa.hsa_get_device_error() == -5
     _no_device_error(hsa)
 
 
