@@ -4,8 +4,9 @@ workspace: it serves callers that cannot allocate device memory themselves
 loop that must not call cudaMalloc because it can synchronise the device).
 
 Through the C ABI it must give exactly what hsa_partition gives with a
-caller-provided workspace, on two calls in a row (the second with a smaller
-input, so anything left in the shared scratch by the first call would show),
+caller-provided workspace, on calls in a row (the second with a smaller
+input, so anything left in the shared scratch by the first call would show,
+the third at a size served by another partition path),
 and it must refuse inputs larger than its fixed scratch before launching.
 This file is collected last on purpose.
 """
@@ -67,6 +68,15 @@ def test_static_partition_matches_workspace_partition_twice(hsa):
     got2 = _static_c_abi(hsa, stat2, 20, budgets2, counts2)
     torch.cuda.synchronize()
     assert torch.equal(got2, ref2)
+
+    # third call: a size the one-block boundary select serves
+    N3 = 30000
+    stat3 = synth.lognormal_stat(N3, 1.0, 5).cuda()
+    budgets3, counts3 = (40, 20, 10, 5), (7000, 8000, 9000, 6000)
+    ref3 = _with_workspace(hsa, stat3, 40, budgets3, counts3)
+    got3 = _static_c_abi(hsa, stat3, 40, budgets3, counts3)
+    torch.cuda.synchronize()
+    assert torch.equal(got3, ref3)
     assert hsa.hsa_get_device_error() == 0
 
 
