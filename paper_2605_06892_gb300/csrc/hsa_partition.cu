@@ -3,12 +3,18 @@
 // caching window).
 //
 // Partition = a stable rank of the statistic.  Each fp32 value is mapped to an
-// unsigned key whose integer order is the float order (-0 folded onto +0), and
-// the (key, token) pairs are sorted by a least-significant-digit radix sort:
-// four passes of 8 bits, each pass a per-tile histogram, one exclusive scan of
-// the (digit, tile) counts in digit-major order, and a stable scatter.  Since
-// every pass is stable and the pairs start in token order, equal statistics
-// stay in token order, which is the tie rule.  Rank r then maps to its group.
+// unsigned key whose integer order is the float order (-0 folded onto +0); the
+// rank of a token is its position in the (key, token) order, which is the tie
+// rule, and rank r maps to its group.  Three paths give the same groups:
+//   N <= 12032   one launch ranks every token by counting the pairs before it;
+//   N <= 49152   one block finds the pair at each group boundary (radix select
+//                over keys held in shared memory) and compares every token with
+//                those pairs;
+//   larger N     a least-significant-digit radix sort of the (key, token)
+//                pairs: four passes of 8 bits, each a per-tile histogram, one
+//                exclusive scan of the (digit, tile) counts in digit-major
+//                order, and a stable scatter (the pairs start in token order,
+//                so equal keys stay in token order), then rank -> group.
 //
 // The active set needs no workspace: block b owns one chunk of tokens, counts
 // the active tokens of all earlier chunks itself (an L2-resident re-read that
