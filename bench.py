@@ -24,6 +24,8 @@ collective on the data path); the timing is the max over ranks.
 from __future__ import annotations
 
 import argparse
+import concurrent.futures as cf
+import dataclasses
 import hashlib
 import json
 import os
@@ -41,6 +43,10 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 METRIC = "HSA active-attention TFLOP/s vs BF16 peak; KV-sync/Euler HBM GB/s"
+# The largest workload that fits one GPU: the full 40-iteration schedule of the
+# 720p Wan-14B layer.  The others run briefly after it (config.also).
+HEADLINE = "wan14b_720p"
+ALSO = ("wan13b", "wan14b_boxes", "ltx", "tiny_f32")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
 
@@ -48,15 +54,30 @@ L2_FLUSH_BYTES = 256 << 20
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="hsa", choices=["hsa", "reference"])
-    p.add_argument("--workload", default="wan13b", choices=list(synth.WORKLOADS))
+    p.add_argument("--workload", default=HEADLINE, choices=list(synth.WORKLOADS))
+    p.add_argument("--heads", type=int, default=0,
+                   help="override the workload's head count (small cases for ncu captures)")
+    p.add_argument("--iters", default="",
+                   help="override the measured iterations, e.g. 0,4,2,1")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-also", action="store_true",
+                   help="skip the short runs of the other workloads (config.also)")
     p.add_argument("--memory-sweep", action="store_true",
                    help="HBM size sweep of gather, KV scatter and cached Euler (L2 flushed)")
     return p.parse_args()
+
+
+def workload_of(args) -> synth.Workload:
+    w = synth.WORKLOADS[args.workload]
+    if args.heads:
+        w = dataclasses.replace(w, H=args.heads)
+    if args.iters:
+        w = dataclasses.replace(w, iters=tuple(int(x) for x in args.iters.split(",")))
+    return w
 
 
 # ------------------------------------------------------------ distributed
@@ -157,36 +178,38 @@ class ClockSampler:
 
 # --------------------------------------------------------------- workload
 
+def host_inputs(w: synth.Workload, rep: int = 0):
+    """The workload's seeded host tensors: hidden rows, Q, K/V cache, fresh K/V,
+    latent, velocity cache, fresh velocities (multi-GB shapes drawn in blocks
+    on the host cores, synth.normal_blocks)."""
+    seed = lambda t: synth.seed_for(w.cid, rep, t)  # noqa: E731
+    dt = w.dtype
+    N, H, D, C = w.N, w.H, w.D, w.C
+    big = lambda shape, t: synth.normal_blocks(shape, seed(t), dt)  # noqa: E731
+    return {"hidden": big((N, H * D), 1), "q": big((N, H, D), 2), "kc": big((N, H, D), 3),
+            "vc": big((N, H, D), 4), "kf": big((N, H, D), 5), "vf": big((N, H, D), 6),
+            "x": synth.normal((N, C), seed(7)), "vh": synth.normal((N, C), seed(8)),
+            "v_fresh": synth.normal((N, C), seed(9))}
+
+
 class Layer:
     """Resident device state and inputs of one HSA layer workload."""
 
-    def __init__(self, w: synth.Workload, dev, rep: int = 0):
+    def __init__(self, w: synth.Workload, dev, rep: int = 0, keep_host: bool = False):
         self.w, self.dev = w, dev
-        N, H, D, C = w.N, w.H, w.D, w.C
+        N, H, D = w.N, w.H, w.D
         self.stat_h, self.counts = synth.stat_for(w, rep)
-        seed = lambda t: synth.seed_for(w.cid, rep, t)  # noqa: E731
-        dt = w.dtype
+        host = host_inputs(w, rep)
+        self.host = host if keep_host else None
         self.stat = self.stat_h.to(dev)
-        self.hidden = synth.normal((N, H * D), seed(1), dt).to(dev)
-        self.q = synth.normal((N, H, D), seed(2), dt).to(dev)
-        self.kc = synth.normal((N, H, D), seed(3), dt).to(dev)
-        self.vc = synth.normal((N, H, D), seed(4), dt).to(dev)
-        self.kf = synth.normal((N, H, D), seed(5), dt).to(dev)
-        self.vf = synth.normal((N, H, D), seed(6), dt).to(dev)
-        self.x = synth.normal((N, C), seed(7)).to(dev)
-        self.vh = synth.normal((N, C), seed(8)).to(dev)
-        self.v_fresh = synth.normal((N, C), seed(9)).to(dev)
+        for k, t in host.items():
+            setattr(self, k, t.to(dev))
         self.group_of = torch.empty(N, dtype=torch.int32, device=dev)
         self.idx = torch.empty(N, dtype=torch.int32, device=dev)
         self.pos = torch.empty(N, dtype=torch.int32, device=dev)
         self.gathered = torch.empty((N, H * D), dtype=self.hidden.dtype, device=dev)
         self.out = torch.empty((N, H, D), dtype=self.q.dtype, device=dev)
         self.iters = list(w.iters)
-
-    def bytes_resident(self):
-        return sum(t.numel() * t.element_size() for t in
-                   (self.hidden, self.q, self.kc, self.vc, self.kf, self.vf, self.x, self.vh,
-                    self.v_fresh, self.gathered, self.out))
 
 
 def algorithmic(w, n_act):
@@ -204,14 +227,83 @@ def algorithmic(w, n_act):
     }
 
 
+def representative_iters(w, counts):
+    """First iteration of each distinct active-set size, in schedule order
+    (the CPU legs' sample of the schedule)."""
+    import oracle
+    seen, out = set(), []
+    for it in w.iters:
+        n = oracle.active_count(w.budgets, counts, w.T, it, w.window_pct)
+        if n not in seen:
+            seen.add(n)
+            out.append(it)
+    return out
+
+
 # ---------------------------------------------------------------- hsa arm
 
 def run_hsa(args, dist, rank, world, local_rank):
     import paper_2605_06892_gb300 as hsa
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    w = synth.WORKLOADS[args.workload]
-    L = Layer(w, dev)
+    w = workload_of(args)
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    L = Layer(w, dev, keep_host=want_cpu)
+    peaks, peak_src = load_peaks()
+    res = measure(args, hsa, L, dev, dist, world, local_rank, args.steps, peaks)
+    flops_step, ms_per_step = res["flops_step"], res["ms_per_step"]
+    value = world * flops_step / (ms_per_step * 1e-3) / 1e12
+    kernels = res["kernels"]
+    att_tflops = kernels["attention"]["tflops"]
+    clocks = res["clocks"]
+    # Peak for the roofline: the measured burst figure for a kernel that runs in
+    # short steps, the sustained one (seconds-long loop under the power cap) for
+    # a kernel timed inside a step that keeps the GPU busy for about a second.
+    long_step = ms_per_step >= 500.0
+    peak = peaks["bf16_tflops_sustained"] if long_step else peaks["bf16_tflops"]
+    roofline = {
+        "bound": "tensor", "achieved": att_tflops, "peak": peak, "unit": "TFLOP/s",
+        "frac": att_tflops / peak, "traffic": profiled_traffic(w, res["n_of"]),
+        "peak_source": (f"{peak_src} bf16 sustained (kernel timed inside a "
+                        f"{ms_per_step / 1e3:.2f} s step)" if long_step
+                        else f"{peak_src} bf16 burst"),
+        "frac_burst": att_tflops / peaks["bf16_tflops"],
+        "frac_sustained": att_tflops / peaks["bf16_tflops_sustained"],
+        "clock_normalised": clock_normalised(att_tflops, clocks, peaks),
+    }
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) Q/K/V, lognormal statistic; no model weights)",
+        "config": {"workload": workload_desc(w, L.counts),
+                   "iterations": res["iterations"], "parallelism": f"replicas x{world}",
+                   "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
+                   "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
+        "kernels": kernels, "roofline": roofline, "dense_baseline": res["dense_baseline"],
+        "gpu_launches": res["launches"],
+        "clocks": clocks,
+    }
+    if not args.no_e2e:
+        line["e2e"] = run_e2e(args, hsa, L, res["sig"], res["n_of"], torch.cuda.current_stream(dev),
+                              dev, dist, world, flops_step, local_rank)
+    if want_cpu:
+        line["cpu_baseline"] = cpu_baseline(w, L)
+    host = L.host
+    del L, host
+    torch.cuda.empty_cache()
+    if not args.no_also and not args.heads and not args.iters and args.workload == HEADLINE:
+        line["config"]["also"] = run_also(args, hsa, dev, dist, world, local_rank, peaks)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
+    """Warm-up, then `steps` timed steps of the workload's hot path (CUDA
+    events on the launching stream, L2 flushed between steps, clocks sampled),
+    then the dense all-token iteration.  Returns the per-kernel and per-step
+    figures."""
+    w = L.w
     T, budgets = w.T, w.budgets
     sig = hsa.hsa_sigma_schedule(T, w.shift)
     ws = torch.empty(hsa.hsa_partition_workspace_bytes(w.N), dtype=torch.uint8, device=dev)
@@ -263,7 +355,7 @@ def run_hsa(args, dist, rank, world, local_rank):
     torch.cuda.synchronize()
     launches0 = hsa.hsa_launch_count()
     with ClockSampler(local_rank) as clocks:
-        for _ in range(args.steps):
+        for _ in range(steps):
             flush.zero_()                       # L2 flush, outside the step's events
             s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             s0.record(stream)
@@ -275,18 +367,14 @@ def run_hsa(args, dist, rank, world, local_rank):
     barrier(dist)
     step_ms = [a.elapsed_time(b) for a, b in step_events]
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
-    ms_per_step = total_ms / args.steps
-    kern_ms = {k: sum(a.elapsed_time(b) for a, b in v) / args.steps for k, v in per_kernel.items()}
+    ms_per_step = total_ms / steps
+    kern_ms = {k: sum(a.elapsed_time(b) for a, b in v) / steps for k, v in per_kernel.items()}
     status = hsa.hsa_get_device_error(stream)
     assert status == 0, f"device error {status}"
 
     flops_step = sum(algorithmic(w, n_of[it])["attention_flops"] for it in L.iters)
-    value = world * flops_step / (ms_per_step * 1e-3) / 1e12
-
-    # memory-bound kernels: algorithmic bytes per step / time per step
     bytes_step = {k: sum(algorithmic(w, n_of[it])[k] for it in L.iters)
                   for k in ("gather", "scatter", "euler", "active")}
-    peaks, peak_src = load_peaks()
     kernels = {
         "attention": {"ms": kern_ms["attention"],
                       "tflops": flops_step / (kern_ms["attention"] * 1e-3) / 1e12},
@@ -303,47 +391,89 @@ def run_hsa(args, dist, rank, world, local_rank):
     att_ms = [0.0] * n_it
     for kind in ("active", "gather", "scatter", "attention", "euler"):
         for e, (a, b) in enumerate(per_kernel[kind]):
-            t = a.elapsed_time(b) / args.steps
+            t = a.elapsed_time(b) / steps
             it_ms[e % n_it] += t
             if kind == "attention":
                 att_ms[e % n_it] += t
     dense = dense_iteration(args, hsa, L, sig, flush, ws_att, stream)
-    per_iter = {}
+    by_frac = {}
     for m, it in enumerate(L.iters):
-        per_iter[str(it)] = {"n_active": n_of[it], "frac": n_of[it] / w.N, "ms": it_ms[m],
-                             "attention_ms": att_ms[m], "vs_dense": it_ms[m] / dense["ms"]}
+        f = round(n_of[it] / w.N, 4)
+        d = by_frac.setdefault(f, {"n_active": n_of[it], "iterations": [], "ms": [],
+                                   "attention_ms": []})
+        d["iterations"].append(it)
+        d["ms"].append(it_ms[m])
+        d["attention_ms"].append(att_ms[m])
+    iterations = {}
+    for f, d in sorted(by_frac.items(), reverse=True):
+        ms = statistics.mean(d["ms"])
+        iterations[f"{f:g}"] = {
+            "n_active": d["n_active"], "iterations": d["iterations"], "ms": ms,
+            "attention_ms": statistics.mean(d["attention_ms"]), "vs_dense": ms / dense["ms"]}
     dense_baseline = {
         "iteration_ms": dense["ms"], "attention_ms": dense["attention_ms"],
         "step_ms_all_dense": n_it * dense["ms"] + kern_ms["partition"],
         "step_vs_all_dense": ms_per_step / (n_it * dense["ms"] + kern_ms["partition"]),
+        "ideal_vs_all_dense": sum(n_of.values()) / (n_it * w.N),
         "what": f"{n_it} iterations with every token active (same kernels, |A| = N), "
                 "against the measured step; L2 flushed before each dense iteration"}
+    return {"flops_step": flops_step, "ms_per_step": ms_per_step, "kernels": kernels,
+            "iterations": iterations, "dense_baseline": dense_baseline, "launches": launches,
+            "clocks": clocks.summary(), "sig": sig, "n_of": n_of}
 
-    att_tflops = kernels["attention"]["tflops"]
-    roofline = {"bound": "tensor", "achieved": att_tflops, "peak": peaks["bf16_tflops"],
-                "unit": "TFLOP/s", "frac": att_tflops / peaks["bf16_tflops"],
-                "traffic": profiled_traffic(w), "peak_source": f"{peak_src} bf16 burst",
-                "frac_sustained": att_tflops / peaks["bf16_tflops_sustained"]}
 
-    line = {
-        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) Q/K/V, lognormal statistic; no model weights)",
-        "config": {"workload": workload_desc(w, L.counts),
-                   "per_iteration": per_iter, "parallelism": f"replicas x{world}",
-                   "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
-                   "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
-        "kernels": kernels, "roofline": roofline, "dense_baseline": dense_baseline,
-        "gpu_launches": launches,
-        "clocks": clocks.summary(),
-    }
-    if not args.no_e2e:
-        line["e2e"] = run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, L)
-    if rank == 0:
-        print(json.dumps(line), flush=True)
+def clock_normalised(att_tflops, clocks, peaks):
+    """The attention rate against the cuBLAS denominator at equal SM clock, and
+    against the tensor pipe's own rate (8192 bf16 FLOP per clock per SM, dense)
+    at the sampled clock.  The denominators' clock: the median SM clock the
+    peak measurement saw under load (MEASURED_PEAKS.json), which the seconds-
+    long sustained loop dominates."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            peak_mhz = float(json.load(f)["clocks_under_load"]["sm_mhz_median"])
+    except (OSError, KeyError, ValueError, TypeError):
+        peak_mhz = None
+    if not clocks or not clocks.get("sm_mhz"):
+        return None
+    mhz = clocks["sm_mhz"]
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    out = {"sm_mhz": mhz, "tensor_pipe_peak_tflops_at_clock": 8192 * sms * mhz * 1e6 / 1e12}
+    out["frac_of_tensor_pipe_at_clock"] = att_tflops / out["tensor_pipe_peak_tflops_at_clock"]
+    if peak_mhz:
+        out["cublas_sustained_sm_mhz"] = peak_mhz
+        out["frac_of_cublas_sustained_at_equal_clock"] = (
+            (att_tflops / mhz) / (peaks["bf16_tflops_sustained"] / peak_mhz))
+    return out
+
+
+def run_also(args, hsa, dev, dist, world, local_rank, peaks):
+    """Short runs of the other workloads (no e2e, no CPU leg): their step rate,
+    attention rate and roofline fraction, memory-kernel fractions and the
+    iteration time against the dense iteration."""
+    out = {}
+    for name in ALSO:
+        w = synth.WORKLOADS[name]
+        L = Layer(w, dev)
+        steps = max(3, min(args.steps, 10))
+        res = measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks)
+        att = res["kernels"]["attention"]["tflops"]
+        out[name] = {
+            "workload": workload_desc(w, L.counts), "steps": steps,
+            "ms_per_step": res["ms_per_step"],
+            "value": world * res["flops_step"] / (res["ms_per_step"] * 1e-3) / 1e12,
+            "attention_tflops": att,
+            "attention_frac_burst": att / peaks["bf16_tflops"] if w.dtype == "bf16" else None,
+            "gather_frac_hbm": res["kernels"]["gather"]["frac_hbm"],
+            "scatter_frac_hbm": res["kernels"]["scatter"]["frac_hbm"],
+            "euler_frac_hbm": res["kernels"]["euler"]["frac_hbm"],
+            "partition_ms": res["kernels"]["partition"]["ms"],
+            "iterations_vs_dense": {f: d["vs_dense"] for f, d in res["iterations"].items()},
+            "step_vs_all_dense": res["dense_baseline"]["step_vs_all_dense"],
+            "gpu_launches": res["launches"], "clocks": res["clocks"]}
+        del L
+        torch.cuda.empty_cache()
+    return out
 
 
 def dense_iteration(args, hsa, L, sig, flush, ws_att, stream, reps=None):
@@ -378,7 +508,7 @@ def dense_iteration(args, hsa, L, sig, flush, ws_att, stream, reps=None):
             "attention_ms": sum(x.elapsed_time(y) for x, y in att) / reps}
 
 
-def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
+def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step, local_rank=0):
     """Same step through the C ABI with host buffers (pinned).  Copies run on
     their own streams and overlap the kernels: each iteration's inputs are
     copied in two iterations ahead into a ring of three device buffers (so a
@@ -487,22 +617,25 @@ def run_e2e(args, hsa, L, sig, n_of, stream, dev, dist, world, flops_step):
     torch.cuda.synchronize()
     barrier(dist)
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(s_in)
-    stream.wait_event(a)
-    s_out.wait_event(a)
-    for _ in range(args.steps):
-        step()
-    s_out.wait_stream(stream)
-    s_out.wait_stream(s_in)
-    b.record(s_out)
-    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks:
+        a.record(s_in)
+        stream.wait_event(a)
+        s_out.wait_event(a)
+        for _ in range(args.steps):
+            step()
+        s_out.wait_stream(stream)
+        s_out.wait_stream(s_in)
+        b.record(s_out)
+        torch.cuda.synchronize()
     barrier(dist)
     ms = max_over_ranks(dist, a.elapsed_time(b), dev) / args.steps
     assert hsa.hsa_get_device_error(stream) == 0
     return {"value": world * flops_step / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
             "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "copies": "pinned host buffers; inputs copied two iterations ahead on a copy "
-                      "stream, outputs copied back on another, overlapping the kernels"}
+                      "stream, outputs copied back on another, overlapping the kernels",
+            "q_load": "compact (the caller copies the active rows' Q; q_idx = NULL)",
+            "clocks": clocks.summary()}
 
 
 def code_digest(text: str) -> str:
@@ -514,74 +647,116 @@ def code_digest(text: str) -> str:
     return hashlib.sha256(text.encode()).hexdigest()[:16]
 
 
-def profiled_traffic(w):
-    """DRAM bytes per attention launch from the committed ncu summary, if it
-    was taken on the current attention code (comments aside); else None."""
+def profiled_traffic(w, n_of):
+    """DRAM bytes per attention launch (read + write), averaged over the step's
+    launches, from the committed ncu summary of this workload's attention
+    kernel, if it was taken on the current attention code (comments aside);
+    else None.  The summary lists bytes per launch at each active fraction,
+    per head (`traffic_per_head_bytes <frac>: <bytes>`), measured on a case
+    with fewer heads; heads are independent, so a launch's traffic scales with
+    H."""
     path = os.path.join(ROOT, "profiles", f"attention_{w.name}.md")
     src = os.path.join(ROOT, "paper_2605_06892_gb300", "csrc", "hsa_attention.cu")
     try:
         digest = code_digest(open(src).read())
-        fields = {}
+        per_head, sha = {}, None
         for line in open(path):
-            if line.startswith("traffic_per_launch_bytes:") or line.startswith("code_sha256:"):
+            if line.startswith("code_sha256:"):
+                sha = line.split(":", 1)[1].strip()
+            elif line.startswith("traffic_per_head_bytes"):
                 k, v = line.split(":", 1)
-                fields[k.strip()] = v.strip()
-        if fields.get("code_sha256") == digest:
-            return float(fields["traffic_per_launch_bytes"])
-    except (OSError, KeyError, ValueError):
-        pass
-    return None
+                per_head[round(float(k.split()[1]), 4)] = float(v)
+        if sha != digest or not per_head:
+            return None
+        tot = 0.0
+        for it, n in n_of.items():
+            f = round(n / w.N, 4)
+            if f not in per_head:
+                return None
+            tot += per_head[f] * w.H
+        return tot / len(n_of)
+    except (OSError, KeyError, ValueError, IndexError):
+        return None
 
 
 # ----------------------------------------------------------- CPU oracle leg
 
-def _oracle_sample(w, stat, counts, tensors, rows_per_iter, iters):
+def host_cores() -> int:
+    return max(1, len(os.sched_getaffinity(0)))
+
+
+def _oracle_sample(w, stat, counts, t, rows_per_iter, iters, threads):
     """The oracle's pass over one bounded sample of the workload: partition,
-    active set, gather, scatter and cached Euler at full size, attention for
-    `rows_per_iter` active query rows (all heads, all N keys) per iteration.
-    Returns (seconds, attention FLOPs done)."""
+    then for each iteration in `iters` the active set, gather, KV scatter and
+    cached Euler at full size, and attention of `rows_per_iter` active query
+    rows (all heads, all N keys).  With threads > 1 the same oracle calls run
+    on disjoint slices (rows of the gather and scatter, tokens of the Euler
+    step, query rows of the attention) in a thread pool; ctypes releases the
+    GIL during each call.  Returns (seconds, attention FLOPs done)."""
     import oracle
-    hidden, q, kc, vc, kf, vf, x, vh, vfr = tensors
     sig = oracle.sigmas(w.T, w.shift)
+    pool = cf.ThreadPoolExecutor(max_workers=threads) if threads > 1 else None
+
+    def run(fn, parts):
+        if pool is None:
+            for p in parts:
+                fn(p)
+        else:
+            list(pool.map(fn, parts))
+
+    def cuts(n):
+        k = max(1, min(threads, n))
+        return [(n * i // k, n * (i + 1) // k) for i in range(k)]
+
     t0 = time.perf_counter()
     g = oracle.partition(stat, w.T, w.budgets, counts)
     flops = 0.0
     for it in iters:
         idx, pos = oracle.active_set(g, w.T, w.budgets, it, w.window_pct)
         n = idx.numel()
-        oracle.gather(hidden, idx)
-        oracle.kv_scatter(kc, vc, kf[:n], vf[:n], idx)
+        run(lambda c: oracle.gather(t["hidden"], idx[c[0]:c[1]]), cuts(n))
+        run(lambda c: oracle.kv_scatter(t["kc"], t["vc"], t["kf"][c[0]:c[1]],
+                                        t["vf"][c[0]:c[1]], idx[c[0]:c[1]]), cuts(n))
         rows = idx[:rows_per_iter]
-        oracle.attention(q, kc, vc, q_idx=rows)
+        run(lambda c: oracle.attention(t["q"], t["kc"], t["vc"], q_idx=rows[c[0]:c[1]]),
+            cuts(rows.numel()))
         flops += 4.0 * rows.numel() * w.N * w.D * w.H
-        oracle.cached_euler_f32(x, vh, vfr[:n], pos, float(sig[it + 1] - sig[it]))
-    return time.perf_counter() - t0, flops
+        ds = float(sig[it + 1] - sig[it])
+        vfr = t["v_fresh"][:n]
+        run(lambda c: oracle.cached_euler_f32(t["x"][c[0]:c[1]], t["vh"][c[0]:c[1]], vfr,
+                                              pos[c[0]:c[1]], ds), cuts(w.N))
+    el = time.perf_counter() - t0
+    if pool is not None:
+        pool.shutdown()
+    return el, flops
 
 
-def _host_tensors(w, rep=0):
-    seed = lambda t: synth.seed_for(w.cid, rep, t)  # noqa: E731
-    dt = w.dtype
-    N, H, D, C = w.N, w.H, w.D, w.C
-    return (synth.normal((N, H * D), seed(1), dt), synth.normal((N, H, D), seed(2), dt),
-            synth.normal((N, H, D), seed(3), dt), synth.normal((N, H, D), seed(4), dt),
-            synth.normal((N, H, D), seed(5), dt), synth.normal((N, H, D), seed(6), dt),
-            synth.normal((N, C), seed(7)), synth.normal((N, C), seed(8)),
-            synth.normal((N, C), seed(9)))
+def _sample_text(w, rows, iters, threads, secs):
+    return (f"partition, then for iterations {iters} (one per distinct active-set size of "
+            f"the schedule) active set, gather, KV scatter and cached Euler at full size "
+            f"plus attention of {rows} active query rows x {w.H} heads x {w.N} keys per "
+            f"iteration; fp64 oracle, {threads} thread(s), {secs:.1f} s")
 
 
-def cpu_baseline(w, L=None, target_s=15.0):
-    """Oracle timed on the host cores on a bounded sample (single thread)."""
-    stat, counts = synth.stat_for(w)
-    tensors = _host_tensors(w)
-    t1, f1 = _oracle_sample(w, stat, counts, tensors, 1, w.iters[:1])
-    per_row = t1 / max(f1, 1.0)
-    rows = max(1, int(target_s / max(per_row * 4.0 * w.N * w.D * w.H, 1e-9) / len(w.iters)))
-    t, f = _oracle_sample(w, stat, counts, tensors, rows, w.iters)
-    return {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
-            "sample": f"partition, active sets, gather, KV scatter and cached Euler at full "
-                      f"size plus attention of {rows} active query rows x {w.H} heads x "
-                      f"{w.N} keys in each of iterations {list(w.iters)}, fp64, "
-                      f"{t:.1f} s single-threaded"}
+def cpu_baseline(w, L, target_mt_s=10.0):
+    """The oracle timed on the host cores on a bounded sample of the workload:
+    all cores (the oracle's own calls on disjoint slices in a thread pool) and,
+    beside it, a single thread on the schedule's first iteration."""
+    counts = L.counts
+    t = L.host
+    stat = L.stat_h
+    iters = representative_iters(w, counts)
+    cores = host_cores()
+    st_t, st_f = _oracle_sample(w, stat, counts, t, 1, iters[:1], 1)
+    # st_t bounds one query row's time from above (it includes the full-size
+    # gather, scatter and Euler of the iteration)
+    per_thread = max(1, int(target_mt_s / max(st_t, 1e-6) / len(iters)))
+    mt_rows = cores * per_thread
+    mt_t, mt_f = _oracle_sample(w, stat, counts, t, mt_rows, iters, cores)
+    return {"value": mt_f / mt_t / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+            "sample": _sample_text(w, mt_rows, iters, cores, mt_t),
+            "single_thread": {"value": st_f / st_t / 1e12, "unit": "TFLOP/s", "cores": 1,
+                              "sample": _sample_text(w, 1, iters[:1], 1, st_t)}}
 
 
 def workload_desc(w, counts) -> str:
@@ -593,31 +768,36 @@ def workload_desc(w, counts) -> str:
 
 def run_reference(args, dist, rank, world):
     """The oracle as the reference arm: each step is a bounded sample of the
-    workload (4 query rows per iteration), timed on the host cores."""
+    workload (partition, then one of the schedule's distinct iterations in turn
+    at full size, with one attention query row per host core), timed on the
+    host cores."""
     if rank != 0:
         return
-    w = synth.WORKLOADS[args.workload]
+    w = workload_of(args)
     stat, counts = synth.stat_for(w)
-    tensors = _host_tensors(w)
-    rows = 4
-    for _ in range(args.warmup):
-        _oracle_sample(w, stat, counts, tensors, rows, w.iters)
+    t = host_inputs(w)
+    iters = representative_iters(w, counts)
+    cores = host_cores()
+    rows = cores
+    # step k samples iteration iters[k mod len(iters)]
+    for k in range(args.warmup):
+        _oracle_sample(w, stat, counts, t, rows, [iters[k % len(iters)]], cores)
     tot_t, tot_f = 0.0, 0.0
-    for _ in range(args.steps):
-        t, f = _oracle_sample(w, stat, counts, tensors, rows, w.iters)
-        tot_t += t
+    for k in range(args.steps):
+        el, f = _oracle_sample(w, stat, counts, t, rows, [iters[k % len(iters)]], cores)
+        tot_t += el
         tot_f += f
     value = tot_f / tot_t / 1e12
-    sample = (f"oracle pass per step: full-size partition/active set/gather/scatter/Euler and "
-              f"attention of {rows} query rows x {w.H} heads per iteration {list(w.iters)}")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * tot_t / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": workload_desc(w, counts)},
-        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                         "sample": "per step: " + _sample_text(w, rows, iters, cores,
+                                                               tot_t / args.steps)
+                         + " (one of these iterations per step, in turn)"},
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }), flush=True)

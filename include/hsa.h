@@ -128,10 +128,15 @@ int hsa_partition(const float *stat, int N, int T, const int *budgets,
  * The paper has no counterpart; the ranking and group assignment are exactly
  * those of hsa_partition (same arguments, same results).
  * Scratch: a fixed device array inside the library, about 4.3 MB, sized for
- * N <= HSA_PARTITION_STATIC_MAX_TOKENS; every GPU that loads the library
- * holds it until the process exits.  Larger N returns HSA_ERR_UNSUPPORTED
- * before any launch.  Nothing is allocated: no cudaMalloc, cudaFree or
- * allocating library call is made.
+ * N <= HSA_PARTITION_STATIC_MAX_TOKENS; every GPU that loads the library's
+ * partition module holds it until the process exits.  The CUDA runtime
+ * reserves it when that module is loaded on a device: when the library is
+ * loaded if CUDA_MODULE_LOADING=EAGER, otherwise (lazy loading, the default)
+ * at the first partition call or symbol query on that device.  A host
+ * framework that claims all device memory up front should therefore make one
+ * call early, before it does.  Larger N returns HSA_ERR_UNSUPPORTED before any
+ * launch.  Nothing is allocated: no cudaMalloc, cudaFree or allocating
+ * library call is made.
  * The first call on a device looks up the array's device address (a CUDA
  * runtime query) for that device, so make that first call before any stream
  * capture.  Every call on a device shares the one array and finds the last
@@ -210,13 +215,29 @@ int hsa_gather_active(const void *src, size_t row_bytes, int N,
  *   k_cache, v_cache  device, [N, H, D] of dtype, updated in place.
  *   k_fresh, v_fresh  device, [n_active, H, D] of dtype (K/V of A_i).
  *   idx               device, int32 [n_active], distinct values in [0, N)
- *                     (A_i never repeats a token; repeated ids race).
+ *                     (A_i never repeats a token; repeated ids race, and
+ *                     hsa_check_indices detects them).
  * H*D*sizeof(dtype) must be a multiple of 16 bytes and every pointer 16-byte
  * aligned.  An index outside [0, N) skips its row (HSA_ERR_INDEX). */
 int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_fresh,
                         const void *v_fresh, const int32_t *idx, int n_active,
                         int N, int H, int D, hsa_dtype dtype,
                         hsa_stream_t stream);
+
+/* Opt-in check of an index array, for debugging (Sec. 2.2: the groups are
+ * disjoint, so an active set never names a token twice, and the KV scatter
+ * above relies on that).  Reports HSA_ERR_INDEX through hsa_get_device_error
+ * when an entry of idx lies outside [0, N) or a value appears more than once;
+ * the hot-path calls do not make this check themselves.
+ *   idx        device, int32 [n], any order.
+ *   workspace  device, >= hsa_check_indices_workspace_bytes(N) bytes (one
+ *              bit per token), 256-byte aligned; overwritten.  Calls sharing
+ *              one workspace must not overlap on the GPU.
+ * Two launches (clear the bitmap, then mark); returns HSA_ERR_WORKSPACE when
+ * the workspace is missing, too small or misaligned. */
+size_t hsa_check_indices_workspace_bytes(int N);
+int hsa_check_indices(const int32_t *idx, int n, int N, void *workspace,
+                      size_t workspace_bytes, hsa_stream_t stream);
 
 /* Rotary position embedding of the active rows (Sec. 2.3: the positional
  * frequencies are subsampled to match A_i).  The table holds, for every token
@@ -301,8 +322,9 @@ size_t hsa_active_attention_workspace_bytes(int n_active, int N, int H, int D,
  *   v_fresh     device, fp32 [n_active, C] (velocities of A_i) or NULL.
  *   pos         device, int32 [N] (as written by hsa_partition_active) or
  *               NULL; both NULL = no refresh.
- *   n_fresh     rows of v_fresh; a pos value outside [-1, n_fresh) is
- *               treated as -1 and reported as HSA_ERR_INDEX.
+ *   n_fresh     rows of v_fresh; a pos value outside [-1, n_fresh) (above
+ *               the range, or any negative value other than -1) is treated
+ *               as -1 and reported as HSA_ERR_INDEX.
  * C must be a positive multiple of 4 and the pointers 16-byte aligned. */
 int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
                      const int32_t *pos, int n_fresh, int N, int C, float dsigma,

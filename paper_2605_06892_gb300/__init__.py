@@ -22,7 +22,8 @@ __all__ = [
     "hsa_active_count", "hsa_sigma_schedule", "hsa_partition_workspace_bytes",
     "hsa_partition", "hsa_partition_static", "hsa_uniform_stat", "hsa_reserve_first_frame",
     "hsa_reorder_tokens", "hsa_partition_active", "hsa_gather_active",
-    "hsa_kv_sync_scatter", "hsa_rope_table", "hsa_rope_rows", "hsa_kv_sync_scatter_rope",
+    "hsa_kv_sync_scatter", "hsa_check_indices", "hsa_check_indices_workspace_bytes",
+    "hsa_rope_table", "hsa_rope_rows", "hsa_kv_sync_scatter_rope",
     "hsa_active_attention", "hsa_active_attention_prefix",
     "hsa_active_attention_workspace_bytes",
     "hsa_cached_euler", "hsa_cached_euler_l1rel",
@@ -71,6 +72,8 @@ _SIGS = {
     "hsa_active_attention_prefix": ([_c_p, _c_p, _c_int, _c_p, _c_p, _c_int, _c_p, _c_p, _c_int,
                                      _c_int, _c_int, _c_f, _c_p, _c_int, _c_p, _c_sz, _c_p],
                                     _c_int),
+    "hsa_check_indices_workspace_bytes": ([_c_int], _c_sz),
+    "hsa_check_indices": ([_c_p, _c_int, _c_int, _c_p, _c_sz, _c_p], _c_int),
     "hsa_rope_table": ([_c_int, _c_int, _c_int, _c_int, _c_d, _c_p], _c_int),
     "hsa_rope_rows": ([_c_p, _c_p, _c_int, _c_int, _c_int, _c_p, _c_int, _c_p], _c_int),
     "hsa_kv_sync_scatter_rope": ([_c_p, _c_p, _c_p, _c_p, _c_p, _c_int, _c_int, _c_int, _c_int,
@@ -230,6 +233,19 @@ def hsa_kv_sync_scatter(k_cache, v_cache, k_fresh, v_fresh, idx, n_active: int,
     _check(lib().hsa_kv_sync_scatter(_p(k_cache), _p(v_cache), _p(k_fresh), _p(v_fresh),
                                      _p(idx), n_active, N, H, D, _dtype_code(k_cache),
                                      _stream(stream)), "hsa_kv_sync_scatter")
+
+
+def hsa_check_indices_workspace_bytes(N: int) -> int:
+    return lib().hsa_check_indices_workspace_bytes(N)
+
+
+def hsa_check_indices(idx, n: int, N: int, workspace, stream=None) -> None:
+    """Opt-in check of idx[:n]: HSA_ERR_INDEX (via hsa_get_device_error) when an
+    entry is outside [0, N) or repeated; workspace: uint8 device tensor of at
+    least hsa_check_indices_workspace_bytes(N) bytes."""
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().hsa_check_indices(_p(idx), n, N, _p(workspace), ws_bytes, _stream(stream)),
+           "hsa_check_indices")
 
 
 def hsa_rope_table(grid, D: int, theta: float = 10000.0) -> torch.Tensor:

@@ -127,7 +127,7 @@ cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
       p[u] = -1;
       if (pos && e[u] < total) {
         p[u] = __ldg(pos + row[u]);
-        if (p[u] >= n_fresh_rows) {
+        if (p[u] >= n_fresh_rows || p[u] < -1) {   // only -1 means "no fresh row"
           set_error(err, kErrIndex);
           p[u] = -1;
         }
@@ -190,7 +190,7 @@ euler_l1rel_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
     for (int k = 0; k < kL1relRows; ++k) {
       n[k] = n0 + k * step + sub;
       p[k] = (n[k] < N) ? __ldg(pos + n[k]) : -1;
-      if (p[k] >= n_fresh_rows) {
+      if (p[k] >= n_fresh_rows || p[k] < -1) {
         set_error(err, kErrIndex);
         p[k] = -1;
       }
@@ -331,6 +331,36 @@ kv_scatter_rope_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
       }
     }
   }
+}
+
+// Index check (opt-in, for debugging a caller's index arrays): every entry of
+// idx must lie in [0, N) and no value may appear twice.  Sec. 2.2 makes the
+// groups disjoint, so A_i never repeats a token; a repeated id would make the
+// KV scatter race.  One bit per token in a caller workspace, cleared first
+// (bitmap_clear_kernel), then set with atomicOr: an entry that finds its bit
+// already set is a repeat.
+__global__ void __launch_bounds__(kThreads)
+bitmap_clear_kernel(uint4 *__restrict__ bits, long long n_vec) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long v = blockIdx.x * (long long)blockDim.x + threadIdx.x; v < n_vec; v += stride)
+    bits[v] = make_uint4(0u, 0u, 0u, 0u);
+}
+
+__global__ void __launch_bounds__(kThreads)
+check_indices_kernel(const int32_t *__restrict__ idx, long long n, int N,
+                     unsigned *__restrict__ bits, unsigned *err) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  bool bad = false;
+  for (long long j = blockIdx.x * (long long)blockDim.x + threadIdx.x; j < n; j += stride) {
+    const int t = __ldg(idx + j);
+    if (t < 0 || t >= N) {
+      bad = true;
+      continue;
+    }
+    const unsigned bit = 1u << (t & 31);
+    if (atomicOr(bits + (t >> 5), bit) & bit) bad = true;
+  }
+  if (bad) set_error(err, kErrIndex);
 }
 
 // Grid for n_rows rows handled by lane groups of size L: up to 8 blocks of
@@ -505,5 +535,37 @@ extern "C" int hsa_kv_sync_scatter_rope(void *k_cache, void *v_cache, const void
   kv_scatter_rope_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
       (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
       n_active, N, (int)vecs, D, (const float4 *)table, log2i(L), err);
+  return launch_status();
+}
+
+extern "C" size_t hsa_check_indices_workspace_bytes(int N) {
+  if (N <= 0) return 0;
+  return (((size_t)N + 31) / 32 * 4 + 255) / 256 * 256;   // one bit per token, whole uint4s
+}
+
+extern "C" int hsa_check_indices(const int32_t *idx, int n, int N, void *workspace,
+                                 size_t workspace_bytes, hsa_stream_t stream) {
+  if (n < 0 || N < 0) return HSA_ERR_INVALID_ARG;
+  if (n == 0) return HSA_OK;
+  if (!idx) return HSA_ERR_INVALID_ARG;
+  const size_t need = hsa_check_indices_workspace_bytes(N);
+  if (N > 0 && (!workspace || workspace_bytes < need ||
+                (reinterpret_cast<uintptr_t>(workspace) & 255)))
+    return HSA_ERR_WORKSPACE;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  const long long cap = (long long)sm_count() * (2048 / kThreads);
+  const long long n_vec = (long long)(need / 16);
+  long long b0 = (n_vec + kThreads - 1) / kThreads, b1 = (n + kThreads - 1) / kThreads;
+  b0 = b0 < 1 ? 1 : (b0 > cap ? cap : b0);
+  b1 = b1 > cap ? cap : b1;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (n_vec > 0) {
+    count_launches(1);
+    bitmap_clear_kernel<<<(int)b0, kThreads, 0, s>>>(static_cast<uint4 *>(workspace), n_vec);
+  }
+  count_launches(1);
+  check_indices_kernel<<<(int)b1, kThreads, 0, s>>>(idx, n, N, static_cast<unsigned *>(workspace),
+                                                    err);
   return launch_status();
 }

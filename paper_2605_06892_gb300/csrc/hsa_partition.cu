@@ -40,15 +40,17 @@ struct GroupStarts {
   int count[kMaxGroups];
 };
 
-size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+constexpr size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
 struct SortLayout {
   size_t keys0, keys1, vals0, vals1, hist, total;
   int tiles;
 };
 
-SortLayout sort_layout(int N) {
-  SortLayout L;
+// Workspace layout of the radix-sort path; constexpr so that the fixed
+// scratch array of hsa_partition_static is sized by this same formula.
+constexpr SortLayout sort_layout(int N) {
+  SortLayout L{};
   L.tiles = (N + kTile - 1) / kTile;
   const size_t a = align256((size_t)N * 4);
   L.keys0 = 0;
@@ -732,11 +734,8 @@ __global__ void reserve_frame_kernel(float *__restrict__ stat, int frame_tokens)
 
 namespace {
 
-constexpr size_t static_workspace_bytes(size_t n) {
-  return 4 * ((n * 4 + 255) / 256 * 256) + ((256 * ((n + kTile - 1) / kTile) * 4 + 255) / 256 * 256);
-}
-
-constexpr size_t kStaticScratchBytes = static_workspace_bytes(HSA_PARTITION_STATIC_MAX_TOKENS);
+constexpr size_t kStaticScratchBytes = sort_layout(HSA_PARTITION_STATIC_MAX_TOKENS).total;
+static_assert(kStaticScratchBytes % 256 == 0, "scratch array size");
 
 // The host cannot use this symbol as a device address; the set-up below asks
 // the runtime for the device address once per device.

@@ -25,7 +25,7 @@ from dataclasses import dataclass, field
 import torch
 
 __all__ = [
-    "Workload", "WORKLOADS", "normal", "lognormal_stat", "box_stat",
+    "Workload", "WORKLOADS", "normal", "normal_blocks", "lognormal_stat", "box_stat",
     "uniform_subset", "seed_for",
 ]
 
@@ -120,6 +120,33 @@ def normal(shape, seed: int, dtype: str = "f32") -> torch.Tensor:
     if dtype == "f32":
         return x
     raise ValueError(dtype)
+
+
+def normal_blocks(shape, seed: int, dtype: str = "f32", workers: int | None = None,
+                  block: int = 4096) -> torch.Tensor:
+    """i.i.d. N(0,1) host tensor for multi-GB shapes: the first dimension is cut
+    into blocks of ``block`` rows and block b is drawn by its own seeded
+    generator (seed * 1000003 + b), in fp32, rounded to ``dtype``.  The blocks
+    are drawn on ``workers`` threads; the values depend only on the seed and the
+    block size, not on the number of threads.  Same distribution as ``normal``
+    (other values)."""
+    import concurrent.futures as cf
+    import os
+    shape = tuple(shape)
+    tdt = {"bf16": torch.bfloat16, "f32": torch.float32}[dtype]
+    out = torch.empty(shape, dtype=tdt)
+    n = shape[0]
+    n_blocks = (n + block - 1) // block
+
+    def fill(b):
+        r0, r1 = b * block, min(n, (b + 1) * block)
+        g = _gen(seed * 1000003 + b)
+        out[r0:r1] = torch.randn((r1 - r0,) + shape[1:], generator=g, dtype=torch.float32)
+
+    workers = workers or max(1, min(32, len(os.sched_getaffinity(0))))
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        list(ex.map(fill, range(n_blocks)))
+    return out
 
 
 def lognormal_stat(N: int, sigma: float, seed: int) -> torch.Tensor:

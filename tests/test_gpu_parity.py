@@ -575,6 +575,63 @@ def test_cached_euler_bad_pos(hsa):
     assert torch.all(x.cpu() == 0.5)
 
 
+@pytest.mark.parametrize("bad", [-2, -5, -(2 ** 31)])
+def test_cached_euler_negative_pos(hsa, bad):
+    """Only -1 means 'no fresh row': any other negative pos is reported as an
+    index error and that token keeps its cached velocity (plain and fused)."""
+    x = torch.zeros((10, 4), device=DEV)
+    vh = torch.ones((10, 4), device=DEV)
+    vfr = torch.full((2, 4), 3.0, device=DEV)
+    pos = torch.full((10,), -1, dtype=torch.int32, device=DEV)
+    pos[1] = 0
+    pos[4] = bad
+    hsa.hsa_cached_euler(x, vh, vfr, pos, 0.5)
+    assert hsa.hsa_get_device_error() == -6
+    exp = torch.full((10, 4), 0.5)
+    exp[1] = 1.5
+    assert torch.equal(x.cpu(), exp)
+    x.zero_()
+    vh.fill_(1.0)
+    stat = torch.zeros(10, device=DEV)
+    hsa.hsa_cached_euler_l1rel(x, vh, vfr, pos, 0.5, stat, 1.0)
+    assert hsa.hsa_get_device_error() == -6
+    assert torch.equal(x.cpu(), exp)
+    assert stat.cpu()[4].item() == 0.0
+
+
+def test_check_indices(hsa):
+    """Opt-in index check: a valid active set passes; a repeated id or one out
+    of range is reported as HSA_ERR_INDEX (Sec. 2.2: groups are disjoint)."""
+    N = 70001
+    ws = torch.empty(hsa.hsa_check_indices_workspace_bytes(N), dtype=torch.uint8, device=DEV)
+    idx = synth.uniform_subset(N, 30000, 5)
+    d = idx.to(DEV)
+    hsa.hsa_check_indices(d, idx.numel(), N, ws)
+    assert hsa.hsa_get_device_error() == 0
+    perm = torch.randperm(N, generator=torch.Generator().manual_seed(3)).to(torch.int32)
+    hsa.hsa_check_indices(perm.to(DEV), N, N, ws)          # a permutation, any order
+    assert hsa.hsa_get_device_error() == 0
+    dup = idx.clone()
+    dup[20000] = dup[123]                                   # one repeated token
+    hsa.hsa_check_indices(dup.to(DEV), dup.numel(), N, ws)
+    assert hsa.hsa_get_device_error() == -6
+    hsa.hsa_check_indices(d, idx.numel(), N, ws)            # the bitmap is cleared per call
+    assert hsa.hsa_get_device_error() == 0
+    oob = idx.clone()
+    oob[-1] = N
+    hsa.hsa_check_indices(oob.to(DEV), oob.numel(), N, ws)
+    assert hsa.hsa_get_device_error() == -6
+    # the active set the library writes passes the check
+    g = torch.randint(0, 3, (N,), generator=torch.Generator().manual_seed(4),
+                      dtype=torch.int32).to(DEV)
+    a_idx = torch.empty(N, dtype=torch.int32, device=DEV)
+    hsa.hsa_partition_active(g, 40, (40, 20, 10), 2, a_idx, None)
+    torch.cuda.synchronize()
+    n = int((g.cpu() <= 1).sum())
+    hsa.hsa_check_indices(a_idx, n, N, ws)
+    assert hsa.hsa_get_device_error() == 0
+
+
 # ------------------------------------------------------- whole schedule
 
 def test_full_schedule_small(hsa):

@@ -601,3 +601,40 @@ def test_rope_rotation_invariants():
     assert abs(float(d1 - d2)) < 0.15
     # the identity row leaves the vector unchanged
     assert torch.equal(rot(a, 0), a)
+
+
+def test_rope_rotation_direction_is_complex_multiplication():
+    """Fixes the rotation convention, which the invariants above leave open
+    (norms and relative dot products hold for either sign): pair (x0, x1) of
+    token n becomes (x0 + i x1) * exp(i * angle), the angle written out here
+    from the band layout, in complex128 (torch), then rounded to bf16."""
+    grid, D, H = (3, 5, 7), 64, 2
+    N = grid[0] * grid[1] * grid[2]
+    tab = oracle.rope_table(grid, D)
+    P, ph = D // 2, D // 6
+    pt = P - 2 * ph
+    x = synth.normal((N, H, D), 21, "bf16")
+    idx = torch.arange(N, dtype=torch.int32)
+    got = oracle.rope_rows(x, idx, tab).double().view(N, H, P, 2)
+    n = torch.arange(N, dtype=torch.float64)
+    f = torch.div(n, grid[1] * grid[2], rounding_mode="floor")
+    hh = torch.div(n, grid[2], rounding_mode="floor") % grid[1]
+    ww = n % grid[2]
+    ang = torch.empty((N, P), dtype=torch.float64)
+    for i in range(P):
+        if i < pt:
+            ang[:, i] = f * 10000.0 ** (-i / pt)
+        elif i < pt + ph:
+            ang[:, i] = hh * 10000.0 ** (-(i - pt) / ph)
+        else:
+            ang[:, i] = ww * 10000.0 ** (-(i - pt - ph) / ph)
+    xc = x.double().view(N, H, P, 2)
+    z = torch.complex(xc[..., 0], xc[..., 1]) * torch.exp(1j * ang)[:, None, :]
+    exp = torch.stack([z.real, z.imag], dim=-1)
+    # bf16 rounding of each output (half an ulp, 2^-9 relative) plus the fp32
+    # table and arithmetic; the opposite rotation misses by 2|x| |sin(angle)|
+    tol = 2.0 ** -8 * exp.abs() + 1e-6
+    assert torch.all((got - exp).abs() <= tol)
+    wrong = torch.complex(xc[..., 0], xc[..., 1]) * torch.exp(-1j * ang)[:, None, :]
+    wrong = torch.stack([wrong.real, wrong.imag], dim=-1)
+    assert ((got - wrong).abs() > tol).float().mean() > 0.5
