@@ -137,7 +137,15 @@ class ClockSampler:
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
                  "--format=csv,noheader,nounits", "-lms", "200"],
                 stdout=self.fh, stderr=subprocess.DEVNULL)
-            time.sleep(0.3)
+            # nvidia-smi's start-up (driver and NVML initialisation) can hold
+            # the GPU for a moment: start timing only once it has written its
+            # first sample (at most 10 s)
+            t0 = time.time()
+            while time.time() - t0 < 10.0 and self.proc.poll() is None:
+                time.sleep(0.05)
+                if os.path.getsize(self.path) > 0:
+                    break
+            time.sleep(0.25)
         except OSError:
             self.proc = None
         return self

@@ -318,6 +318,7 @@ struct TcArgs {
   // key ranges of a tail unit and writes its unnormalised O, running maximum
   // and sum to ws_o / ws_ml for the combine kernel.
   int n_qblocks, n_whole, pieces;
+  int wave;           // CTAs resident at once (one per SM): the length of a wave
   float *ws_o;        // [piece CTA][kQT*kBM rows][D] fp32
   float *ws_ml;       // [piece CTA][kQT*kBM rows][2] fp32: m (log2 units), l
 };
@@ -470,13 +471,20 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   const int row0 = wk.row0;
   const int j0 = wk.j0;
   const int nT = wk.j1 - wk.j0;        // key tiles of this CTA (local index j = 0..nT-1)
+  // Key order of the unit.  Whole units of odd "waves" (blocks [k*sms,
+  // (k+1)*sms) for odd k) walk the keys backwards, so they start on the key
+  // tiles the previous wave's units of the same head read last, which are
+  // still in L2.  The order of the keys does not change the result (up to
+  // rounding): the softmax is accumulated online.
+  const bool rev = wk.piece < 0 && ((blockIdx.x / a.wave) & 1);
+  auto key_tile = [&](int j) { return rev ? wk.j1 - 1 - j : j0 + j; };
 
   // K or V tile L/2 of this unit's key range (L even: K, odd: V) into its
   // ring slot, completing on bar_full.  Issued by thread 0, the producer.
   auto load_kv = [&](int L) {
     const int slot = L % C::kStages;
     mbar_expect_tx(&bar_full[slot], C::kTileBytes);
-    const int jg = j0 + (L >> 1);                   // global key tile
+    const int jg = key_tile(L >> 1);                // global key tile
     const bool second = jg >= a.tiles1;
     const CUtensorMap *map = second ? ((L & 1) ? &tm_v2 : &tm_k2) : ((L & 1) ? &tm_v : &tm_k);
     const int y = (second ? jg - a.tiles1 : jg) * kBN;
@@ -734,7 +742,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err));
       if (ok) {
         fence_after();
-        const int jg = j0 + j;                     // keys of this tile that exist
+        const int jg = key_tile(j);                // keys of this tile that exist
         const int valid = jg < a.tiles1 ? a.rows1 - jg * kBN : a.rows2 - (jg - a.tiles1) * kBN;
         if (valid >= kBN)
           softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
@@ -1031,6 +1039,7 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   const long long units = (long long)a.n_qblocks * H;
   if (units > 0x7fffffffLL) return HSA_ERR_UNSUPPORTED;
   const int sms = sm_count();
+  a.wave = sms;
   const int rem = (int)(units % sms);
   int pieces = 1;
   if (ws && rem > 0) {

@@ -6,20 +6,23 @@
 // unsigned key whose integer order is the float order (-0 folded onto +0); the
 // rank of a token is its position in the (key, token) order, which is the tie
 // rule, and rank r maps to its group.  Three paths give the same groups:
-//   N <= 12032   one launch ranks every token by counting the pairs before it;
-//   N <= 49152   one block finds the pair at each group boundary (radix select
-//                over keys held in shared memory) and compares every token with
-//                those pairs;
-//   larger N     a least-significant-digit radix sort of the (key, token)
-//                pairs: four passes of 8 bits, each a per-tile histogram, one
-//                exclusive scan of the (digit, tile) counts in digit-major
-//                order, and a stable scatter (the pairs start in token order,
-//                so equal keys stay in token order), then rank -> group.
+//   N <= 12032    one launch ranks every token by counting the pairs before it;
+//   N <= 360448   one launch of a cluster of 8 CTAs (keys spread over their
+//                 shared memory) finds the pair at each group boundary by radix
+//                 select and compares every token with those pairs;
+//   larger N      a least-significant-digit radix sort of the (key, token)
+//                 pairs: four passes of 8 bits, each a per-tile histogram, one
+//                 exclusive scan of the (digit, tile) counts in digit-major
+//                 order, and a stable scatter (the pairs start in token order,
+//                 so equal keys stay in token order), then rank -> group.
 //
-// The active set needs no workspace: block b owns one chunk of tokens, counts
-// the active tokens of all earlier chunks itself (an L2-resident re-read that
-// is cheap at the token counts of a video DiT), then compacts its own chunk
-// with warp ballots and a block scan.
+// The active set needs no workspace.  Up to 2097152 tokens one cluster of 8
+// CTAs marks and counts the active tokens of its ranges, exchanges the counts
+// through distributed shared memory and compacts; above that, block b owns one
+// chunk of tokens, counts the active tokens of all earlier chunks itself, then
+// compacts its own chunk with warp ballots and a block scan.
+#include <cooperative_groups.h>
+
 #include <algorithm>
 #include <atomic>
 
@@ -236,20 +239,17 @@ rank_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStarts 
   }
 }
 
-// ------------------------------------------------ mid-size layers: select
+// ------------------------------------------------ larger layers: select
 //
 // A token's group depends only on which group boundaries its rank passes:
 // rank >= start[k] for k = 0 .. K-2 (group K-1 holds the lowest ranks), and
 // rank >= b holds exactly when (key, token) >= the pair of rank b in the
-// (key, token) order.  So for kRankMaxN < N <= kSelectMaxN one block loads the
-// N keys into shared memory, finds the pair of each boundary rank (a radix
-// select: four 8-bit digit passes, each a histogram of the keys that share
-// the boundary's digits so far, then the boundary's position among the keys
-// equal to its key, counted in token order) and compares every token with
-// those pairs.  One launch instead of fourteen, and the same ranks as the
-// stable sort.
-constexpr int kSelectThreads = 1024;
-constexpr int kSelectMaxN = 49152;                     // keys: 192 KB of shared memory
+// (key, token) order.  So it is enough to find the pair of each boundary rank
+// (a radix select: four 8-bit digit passes, each a histogram of the keys that
+// share the boundary's digits so far, then the boundary's position among the
+// keys equal to its key, counted in token order) and to compare every token
+// with those pairs: one launch instead of a sort's fourteen, and the same
+// ranks as the stable sort.
 constexpr int kMaxBounds = kMaxGroups - 1;
 
 __device__ __forceinline__ uint32_t order_key(float f) {
@@ -258,46 +258,60 @@ __device__ __forceinline__ uint32_t order_key(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);     // float order as uint order
 }
 
-__global__ void __launch_bounds__(kSelectThreads)
-select_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStarts gs,
-                        int32_t *__restrict__ group_of, unsigned *err) {
-  extern __shared__ uint4 skey4[];                      // the N keys, padded to whole uint4
-  uint32_t *skey = reinterpret_cast<uint32_t *>(skey4);
-  __shared__ uint32_t hist[kMaxBounds][256];
-  __shared__ uint32_t pre[kMaxBounds];      // boundary key digits found so far
-  __shared__ int below[kMaxBounds];         // keys ordered below that digit prefix
-  __shared__ int slot[kMaxBounds];          // histogram of the boundary's prefix
-  __shared__ uint32_t dpre[kMaxBounds];     // distinct prefixes, ascending
+// The select runs on a thread-block cluster of
+// kCsCtas CTAs (one launch).  CTA c holds the keys of tokens [c*chunk,
+// (c+1)*chunk) in its shared memory; each digit pass builds one histogram per
+// CTA, and every CTA then sums the cluster's histograms through distributed
+// shared memory and takes the same digit decisions (identical integer work on
+// identical data, so no broadcast is needed).  The boundary token is found in
+// the CTA whose token range holds it (counts of equal keys are exchanged the
+// same way, in CTA order = token order); that CTA writes the boundary pair into
+// every CTA's shared memory.  Cluster barriers are hardware barriers: every
+// thread of every CTA reaches each of them, so none can wait forever.
+constexpr int kCsCtas = 8;
+constexpr int kCsThreads = 1024;
+constexpr int kCsMaxChunk = 44 * 1024;                 // keys per CTA: 176 KB
+constexpr int kCsMaxN = kCsCtas * kCsMaxChunk;         // 360448 tokens
+
+__global__ void __cluster_dims__(kCsCtas, 1, 1) __launch_bounds__(kCsThreads, 1)
+cluster_select_kernel(const float *__restrict__ stat, int N, int chunk, int K, GroupStarts gs,
+                      int32_t *__restrict__ group_of, unsigned *err) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  extern __shared__ uint4 ckey4[];                     // this CTA's keys, padded to uint4
+  uint32_t *skey = reinterpret_cast<uint32_t *>(ckey4);
+  __shared__ uint32_t hist[kMaxBounds * 256];          // [prefix slot][digit]
+  __shared__ uint32_t pre[kMaxBounds];                 // boundary key digits found so far
+  __shared__ int below[kMaxBounds];                    // keys ordered below that prefix
+  __shared__ int slot[kMaxBounds];                     // histogram of the boundary's prefix
+  __shared__ uint32_t dpre[kMaxBounds];                // distinct prefixes, ascending
   __shared__ int nd;
-  __shared__ unsigned long long thr[kMaxBounds];   // boundary pair (key << 32 | token)
-  __shared__ int warp_tot[kSelectThreads / 32];
+  __shared__ int eqc[kMaxBounds];                      // local keys equal to a boundary key
+  __shared__ unsigned long long thr[kMaxBounds];       // boundary pair (key << 32 | token)
+  __shared__ int warp_tot[kCsThreads / 32];
+  const int cta = (int)cl.block_rank();
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int nb = K - 1;
-  const int n4 = (N + 3) >> 2;
-  // boundary j is searched when 0 < start[j] < N (rank 0 is passed by every
-  // token, rank N by none)
+  const int lo = min(N, cta * chunk), hi = min(N, lo + chunk);
+  const int n_loc = hi - lo;
+  const int n4 = (n_loc + 3) >> 2;
   auto searched = [&](int j) { return gs.start[j] > 0 && gs.start[j] < N; };
-  if ((reinterpret_cast<uintptr_t>(stat) & 15) == 0) {
-    for (int i = threadIdx.x; i < n4; i += kSelectThreads) {
-      float4 f;
-      if (4 * i + 3 < N) {
-        f = reinterpret_cast<const float4 *>(stat)[i];
-      } else {
-        f.x = stat[4 * i];
-        f.y = 4 * i + 1 < N ? stat[4 * i + 1] : 0.f;
-        f.z = 4 * i + 2 < N ? stat[4 * i + 2] : 0.f;
-        f.w = 0.f;
-      }
-      if (!(isfinite(f.x) && isfinite(f.y) && isfinite(f.z) && isfinite(f.w)))
-        set_error(err, kErrNonfinite);
-      skey4[i] = make_uint4(order_key(f.x), order_key(f.y), order_key(f.z), order_key(f.w));
+
+  // keys of [lo, hi); chunk is a multiple of 4, so a 16-byte aligned stat
+  // gives 16-byte aligned rows
+  const bool vec = (reinterpret_cast<uintptr_t>(stat) & 15) == 0;
+  for (int i = threadIdx.x; i < n4; i += kCsThreads) {
+    float f[4];
+    if (vec && 4 * i + 3 < n_loc) {
+      const float4 v = __ldg(reinterpret_cast<const float4 *>(stat + lo) + i);
+      f[0] = v.x, f[1] = v.y, f[2] = v.z, f[3] = v.w;
+    } else {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) f[e] = 4 * i + e < n_loc ? __ldg(stat + lo + 4 * i + e) : 0.f;
     }
-  } else {
-    for (int n = threadIdx.x; n < 4 * n4; n += kSelectThreads) {
-      const float f = n < N ? stat[n] : 0.f;
-      if (!isfinite(f)) set_error(err, kErrNonfinite);
-      skey[n] = order_key(f);
-    }
+    if (!(isfinite(f[0]) && isfinite(f[1]) && isfinite(f[2]) && isfinite(f[3])))
+      set_error(err, kErrNonfinite);
+    ckey4[i] = make_uint4(order_key(f[0]), order_key(f[1]), order_key(f[2]), order_key(f[3]));
   }
   if (threadIdx.x == 0) {
     nd = 1;
@@ -307,38 +321,54 @@ select_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStart
     pre[threadIdx.x] = 0u;
     below[threadIdx.x] = 0;
     slot[threadIdx.x] = 0;
+    eqc[threadIdx.x] = 0;
   }
   __syncthreads();
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
     const int n_hist = nd;
-    for (int i = threadIdx.x; i < n_hist * 256; i += kSelectThreads) hist[i >> 8][i & 255] = 0u;
+    for (int i = threadIdx.x; i < n_hist * 256; i += kCsThreads) hist[i] = 0u;
     __syncthreads();
-    for (int i = threadIdx.x; i < n4; i += kSelectThreads) {
-      const uint4 k4 = skey4[i];
+    // Local histogram.  Every lane of a warp runs the same number of rounds,
+    // so the warp can merge equal bins (__match_any_sync) and add each bin's
+    // count once: in early passes most keys share a few bins.
+    for (int b4 = 0; b4 < n4; b4 += kCsThreads) {
+      const int i = b4 + threadIdx.x;
+      uint4 k4 = make_uint4(0u, 0u, 0u, 0u);
+      if (i < n4) k4 = ckey4[i];
       const uint32_t kk[4] = {k4.x, k4.y, k4.z, k4.w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        if (4 * i + e >= N) break;                     // padding
-        const uint32_t key = kk[e];
-        const uint32_t hi = pass == 0 ? 0u : key >> (shift + 8);
-        for (int q = 0; q < n_hist; ++q) {             // few distinct prefixes
-          const uint32_t v = dpre[q];
-          if (v >= hi) {
-            if (v == hi) atomicAdd(&hist[q][(key >> shift) & 255u], 1u);
-            break;
+        uint32_t bin = 0xffffffffu;                    // no histogram
+        if (i < n4 && 4 * i + e < n_loc) {
+          const uint32_t key = kk[e];
+          const uint32_t hp = pass == 0 ? 0u : key >> (shift + 8);
+          for (int q = 0; q < n_hist; ++q) {           // few distinct prefixes
+            const uint32_t v = dpre[q];
+            if (v >= hp) {
+              if (v == hp) bin = (uint32_t)q * 256u + ((key >> shift) & 255u);
+              break;
+            }
           }
         }
+        const unsigned peers = __match_any_sync(0xffffffffu, bin);
+        if (bin != 0xffffffffu && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
       }
     }
-    __syncthreads();
-    // warp j picks boundary j's digit: the bin where its rank falls
+    cl.sync();                                         // every CTA's histogram is complete
+    // warp j picks boundary j's digit from the cluster's summed histogram
     if (w < nb && searched(w)) {
       const int target = gs.start[w] - below[w];       // rank among the prefix's keys
-      const uint32_t *h = hist[slot[w]];
       int c[8], sum = 0;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) { c[i] = (int)h[8 * lane + i]; sum += c[i]; }
+      for (int i = 0; i < 8; ++i) c[i] = 0;
+      for (int r = 0; r < kCsCtas; ++r) {
+        const uint32_t *h = cl.map_shared_rank(hist, r) + slot[w] * 256 + 8 * lane;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) c[i] += (int)h[i];
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) sum += c[i];
       int incl = sum;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -363,40 +393,50 @@ select_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStart
       for (int j = 0; j < nb; ++j) {
         if (!searched(j)) continue;
         const uint32_t v = pre[j];
-        int pos = 0;
-        while (pos < m && dpre[pos] < v) ++pos;
-        if (pos == m || dpre[pos] != v) {
-          for (int q = m; q > pos; --q) dpre[q] = dpre[q - 1];
-          dpre[pos] = v;
+        int p = 0;
+        while (p < m && dpre[p] < v) ++p;
+        if (p == m || dpre[p] != v) {
+          for (int q = m; q > p; --q) dpre[q] = dpre[q - 1];
+          dpre[p] = v;
           ++m;
         }
       }
       for (int j = 0; j < nb; ++j) {
         if (!searched(j)) continue;
-        int pos = 0;
-        while (dpre[pos] != pre[j]) ++pos;
-        slot[j] = pos;
+        int p = 0;
+        while (dpre[p] != pre[j]) ++p;
+        slot[j] = p;
       }
       nd = m > 0 ? m : 1;
     }
-    __syncthreads();
+    cl.sync();                // no CTA clears its histogram while another reads it
   }
-  // Boundary j's pair: its key pre[j] and the token of rank start[j] - below[j]
-  // among the tokens with that key in token order.  Thread t counts a
-  // contiguous run of tokens; an odd run length keeps the threads of a warp
-  // on different shared-memory banks.
-  const int run = ((N + kSelectThreads - 1) / kSelectThreads) | 1;
-  const int r0 = min(N, threadIdx.x * run), r1 = min(N, r0 + run);
+  // Keys equal to each boundary key in this CTA: one sweep over a contiguous
+  // run of tokens per thread (an odd run length spreads a warp's reads over
+  // the shared-memory banks).
+  const int run = ((n_loc + kCsThreads - 1) / kCsThreads) | 1;
+  const int r0 = min(n_loc, threadIdx.x * run), r1 = min(n_loc, r0 + run);
   for (int j = 0; j < nb; ++j) {
-    const int b = gs.start[j];
-    if (!searched(j)) {                                // the same for every thread
-      if (threadIdx.x == 0) thr[j] = b <= 0 ? 0ull : ~0ull;
-      continue;
-    }
+    if (!searched(j)) continue;
     const uint32_t kj = pre[j];
     int eq = 0;
     for (int n = r0; n < r1; ++n) eq += skey[n] == kj;
-    // exclusive block sum of eq
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) eq += __shfl_xor_sync(0xffffffffu, eq, o);
+    if (lane == 0 && eq) atomicAdd(&eqc[j], eq);
+  }
+  for (int j = threadIdx.x; j < nb; j += kCsThreads)
+    if (!searched(j)) thr[j] = gs.start[j] <= 0 ? 0ull : ~0ull;
+  cl.sync();                                           // every CTA's eqc is complete
+  for (int j = 0; j < nb; ++j) {
+    if (!searched(j)) continue;                        // the same in every thread
+    int before_cta = 0;                                // equal keys in earlier CTAs
+    for (int r = 0; r < cta; ++r) before_cta += *cl.map_shared_rank(&eqc[j], r);
+    const int need = gs.start[j] - below[j] - before_cta;
+    if (need < 0 || need >= eqc[j]) continue;          // another CTA holds it
+    const uint32_t kj = pre[j];
+    int eq = 0;
+    for (int n = r0; n < r1; ++n) eq += skey[n] == kj;
     int incl = eq;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -417,13 +457,13 @@ select_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStart
     }
     __syncthreads();
     const int before = warp_tot[w] + incl - eq;
-    const int need = b - below[j];
     if (need >= before && need < before + eq) {
       int seen = before;
       for (int n = r0; n < r1; ++n) {
         if (skey[n] != kj) continue;
         if (seen == need) {
-          thr[j] = ((unsigned long long)kj << 32) | (unsigned)n;
+          const unsigned long long pair = ((unsigned long long)kj << 32) | (unsigned)(lo + n);
+          for (int r = 0; r < kCsCtas; ++r) *cl.map_shared_rank(&thr[j], r) = pair;
           break;
         }
         ++seen;
@@ -431,12 +471,12 @@ select_partition_kernel(const float *__restrict__ stat, int N, int K, GroupStart
     }
     __syncthreads();                                   // warp_tot is reused
   }
-  __syncthreads();
-  for (int n = threadIdx.x; n < N; n += kSelectThreads) {
-    const unsigned long long kn = ((unsigned long long)skey[n] << 32) | (unsigned)n;
+  cl.sync();                  // the boundary pairs have reached every CTA
+  for (int n = threadIdx.x; n < n_loc; n += kCsThreads) {
+    const unsigned long long kn = ((unsigned long long)skey[n] << 32) | (unsigned)(lo + n);
     int passed = 0;
     for (int j = 0; j < nb; ++j) passed += kn >= thr[j];
-    group_of[n] = K - 1 - passed;
+    group_of[lo + n] = K - 1 - passed;
   }
 }
 
@@ -517,10 +557,129 @@ active_set_kernel(const int32_t *__restrict__ group_of, int N, int K, uint32_t m
   }
 }
 
+// Active set of layers up to kAcMaxN tokens in one cluster of kCsCtas CTAs:
+// CTA c owns tokens [c*chunk, (c+1)*chunk).  First pass: each CTA marks its
+// active tokens (one bit each, in shared memory) and counts them.  The CTAs
+// exchange their counts through distributed shared memory (CTA order is token
+// order), so CTA c learns how many active tokens come before its range; the
+// second pass compacts from the bits.  Group ids are read once, and no global
+// scratch or inter-CTA spin is needed.
+constexpr int kAcThreads = 1024;
+constexpr int kAcMaxChunk = 256 * 1024;                // tokens per CTA: 32 KB of bits
+constexpr int kAcMaxN = kCsCtas * kAcMaxChunk;         // 2097152 tokens
+
+__global__ void __cluster_dims__(kCsCtas, 1, 1) __launch_bounds__(kAcThreads, 1)
+active_set_cluster_kernel(const int32_t *__restrict__ group_of, int N, int K, uint32_t mask,
+                          int chunk, int32_t *__restrict__ idx, int32_t *__restrict__ pos,
+                          unsigned *err) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  __shared__ uint32_t bits[kAcMaxChunk / 32];          // bit t: token lo + t is active
+  __shared__ int warp_cnt[kAcThreads / 32];
+  __shared__ int cta_count;
+  __shared__ int cta_base;
+  const int cta = (int)cl.block_rank();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int lo = min(N, cta * chunk), hi = min(N, lo + chunk);
+  const int n_loc = hi - lo;
+  const int rounds = (n_loc + kAcThreads - 1) / kAcThreads;
+  auto act = [&](int g) -> int { return (g >= 0 && g < K) ? (int)((mask >> g) & 1u) : 0; };
+  // pass 1: bits and count; four rounds' loads are issued before their ballots
+  int c = 0;
+  for (int r0 = 0; r0 < rounds; r0 += 4) {
+    int g[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int t = (r0 + u) * kAcThreads + threadIdx.x;
+      g[u] = t < n_loc ? __ldg(group_of + lo + t) : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (r0 + u >= rounds) break;                     // uniform across the block
+      const int t = (r0 + u) * kAcThreads + threadIdx.x;
+      int flag = 0;
+      if (t < n_loc) {
+        if (g[u] < 0 || g[u] >= K) set_error(err, kErrIndex);
+        flag = act(g[u]);
+      }
+      const unsigned bal = __ballot_sync(0xffffffffu, flag);
+      if (lane == 0) {
+        bits[(r0 + u) * (kAcThreads / 32) + w] = bal;
+        c += __popc(bal);
+      }
+    }
+  }
+  if (lane == 0) warp_cnt[w] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int s = 0;
+    for (int i = 0; i < kAcThreads / 32; ++i) s += warp_cnt[i];
+    cta_count = s;
+  }
+  cl.sync();                                           // every CTA's count is known
+  if (threadIdx.x == 0) {
+    int b = 0;
+    for (int r = 0; r < cta; ++r) b += *cl.map_shared_rank(&cta_count, r);
+    cta_base = b;
+  }
+  cl.sync();                  // no CTA exits while another still reads its count
+  // pass 2: compact from the bits, one round of kAcThreads tokens at a time
+  int base = cta_base;
+  for (int r = 0; r < rounds; ++r) {
+    const int t = r * kAcThreads + threadIdx.x;
+    const unsigned bal = bits[r * (kAcThreads / 32) + w];
+    int before = 0, total = 0;
+    for (int i = 0; i < kAcThreads / 32; ++i) {
+      const int v = __popc(bits[r * (kAcThreads / 32) + i]);
+      before += (i < w) ? v : 0;
+      total += v;
+    }
+    const int flag = (bal >> lane) & 1u;
+    const int rank = base + before + __popc(bal & ((1u << lane) - 1u));
+    if (t < n_loc) {
+      if (flag) idx[rank] = lo + t;
+      if (pos) pos[lo + t] = flag ? rank : -1;
+    }
+    base += total;
+  }
+}
+
 }  // namespace
 }  // namespace hsa
 
 using namespace hsa;
+
+namespace {
+
+// Opts the cluster kernel in to its shared memory on the current device and
+// checks that one cluster of kCsCtas such CTAs can be resident; otherwise the
+// partition takes the radix-sort path.  Resolved once per device.
+bool cluster_select_ready() {
+  static std::atomic<int> state[64];            // 0 unknown, 1 ready, 2 unavailable
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  int st = state[dev].load();
+  if (st == 0) {
+    st = 2;
+    const int smem = kCsMaxChunk * (int)sizeof(uint32_t);
+    if (cudaFuncSetAttribute(cluster_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(kCsCtas);
+      cfg.blockDim = dim3(kCsThreads);
+      cfg.dynamicSmemBytes = smem;
+      int clusters = 0;
+      if (cudaOccupancyMaxActiveClusters(&clusters, cluster_select_kernel, &cfg) == cudaSuccess &&
+          clusters >= 1)
+        st = 1;
+    }
+    cudaGetLastError();                          // a refused query leaves no sticky error
+    state[dev].store(st);
+  }
+  return st == 1;
+}
+
+}  // namespace
 
 extern "C" size_t hsa_partition_workspace_bytes(int N) {
   if (N <= 0) return 0;
@@ -561,19 +720,11 @@ extern "C" int hsa_partition(const float *stat, int N, int T, const int *budgets
                             (size_t)N * sizeof(uint32_t), s>>>(stat, N, K, gs, group_of, err);
     return launch_status();
   }
-  if (N <= kSelectMaxN) {
-    static std::atomic<int> configured[64];
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return HSA_ERR_CUDA;
-    if (!configured[dev].load()) {
-      if (cudaFuncSetAttribute(select_partition_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               kSelectMaxN * (int)sizeof(uint32_t)) != cudaSuccess)
-        return HSA_ERR_CUDA;
-      configured[dev].store(1);
-    }
+  if (N <= kCsMaxN && cluster_select_ready()) {
+    const int chunk = (((N + kCsCtas - 1) / kCsCtas) + 3) & ~3;   // keys per CTA, whole uint4
     count_launches(1);
-    select_partition_kernel<<<1, kSelectThreads, (size_t)((N + 3) / 4) * sizeof(uint4), s>>>(
-        stat, N, K, gs, group_of, err);
+    cluster_select_kernel<<<kCsCtas, kCsThreads, (size_t)chunk * sizeof(uint32_t), s>>>(
+        stat, N, chunk, K, gs, group_of, err);
     return launch_status();
   }
   const int ew_blocks = (int)std::min<long long>((N + kSortThreads - 1) / kSortThreads,
@@ -611,15 +762,22 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
     const bool full = iter < m || iter > T - m - 1;
     if (full || iter % (T / budgets[k]) == 0) mask |= 1u << k;
   }
-  // Chunks of whole 1024-token rounds, at most one block per SM: a layer of
-  // up to 152 * 1024 tokens is compacted in one round per block.
+  cudaStream_t s = (cudaStream_t)stream;
+  unsigned *err = device_error_word();
+  if (!err) return HSA_ERR_CUDA;
+  if (N <= kAcMaxN) {
+    const int chunk = (N + kCsCtas - 1) / kCsCtas;
+    count_launches(1);
+    active_set_cluster_kernel<<<kCsCtas, kAcThreads, 0, s>>>(group_of, N, K, mask, chunk, idx,
+                                                             pos, err);
+    return launch_status();
+  }
+  // Larger layers: chunks of whole 1024-token rounds, at most one block per
+  // SM; block b counts the active tokens of the chunks before its own.
   const int sms = sm_count();
   long long chunk = ((long long)N + sms - 1) / sms;
   chunk = ((chunk + kActThreads - 1) / kActThreads) * kActThreads;
   const int blocks = (int)(((long long)N + chunk - 1) / chunk);
-  cudaStream_t s = (cudaStream_t)stream;
-  unsigned *err = device_error_word();
-  if (!err) return HSA_ERR_CUDA;
   count_launches(1);
   if (aligned16(group_of))
     active_set_kernel<true><<<blocks, kActThreads, 0, s>>>(group_of, N, K, mask, (int)chunk, idx,

@@ -1,9 +1,10 @@
 """The library's launch counter (hsa_launch_count) on the GPU: each entry point
 adds the number of kernels it enqueues, which is what the bench reports as its
-launch count.  Partition of a layer of at most 49152 tokens is one launch (a
-ranking up to 12032 tokens, then a one-block boundary select); larger layers
-take the 4-pass radix sort (key, then histogram + scan + scatter per pass) plus
-the group assignment.  bf16 attention with a workspace
+launch count.  Partition of a layer of at most 360448 tokens is one launch (a
+ranking up to 12032 tokens, then a boundary select on one cluster of 8 CTAs);
+larger layers take the 4-pass radix sort (key, then histogram + scan + scatter
+per pass) plus the group assignment.  The active set is one launch at any
+size.  bf16 attention with a workspace
 adds a combine launch exactly when its last wave is split along the keys."""
 import pytest
 import torch
@@ -37,10 +38,10 @@ def test_launch_counts(hsa):
     stat = synth.lognormal_stat(N, 1.0, 3).to(DEV)
     g = torch.empty(N, dtype=torch.int32, device=DEV)
     ws = torch.empty(hsa.hsa_partition_workspace_bytes(N), dtype=torch.uint8, device=DEV)
-    # up to 49152 tokens the partition takes one launch (rank by count, then
-    # boundary select); beyond, the radix sort takes fourteen
+    # up to 360448 tokens the partition takes one launch (rank by count, then
+    # the cluster boundary select); beyond, the radix sort takes fourteen
     assert _delta(hsa, lambda: hsa.hsa_partition(stat, T, budgets, counts, g, ws)) == 1
-    for Nb, launches in ((20000, 1), (300000, 14)):
+    for Nb, launches in ((20000, 1), (75600, 1), (360448, 1), (360449, 14)):
         stat_b = synth.lognormal_stat(Nb, 1.0, 4).to(DEV)
         g_b = torch.empty(Nb, dtype=torch.int32, device=DEV)
         ws_b = torch.empty(hsa.hsa_partition_workspace_bytes(Nb), dtype=torch.uint8, device=DEV)
@@ -50,6 +51,10 @@ def test_launch_counts(hsa):
     idx = torch.empty(N, dtype=torch.int32, device=DEV)
     pos = torch.empty(N, dtype=torch.int32, device=DEV)
     assert _delta(hsa, lambda: hsa.hsa_partition_active(g, T, budgets, 0, idx, pos)) == 1
+    Nl = 2097153                                     # above the one-cluster active set
+    g_l = torch.zeros(Nl, dtype=torch.int32, device=DEV)
+    i_l = torch.empty(Nl, dtype=torch.int32, device=DEV)
+    assert _delta(hsa, lambda: hsa.hsa_partition_active(g_l, T, budgets, 1, i_l, None)) == 1
     n = N
     rows = synth.normal((N, H * D), 1, "bf16").to(DEV)
     out = torch.empty_like(rows)

@@ -81,15 +81,18 @@ def test_partition_ties_signed_zero_ragged(hsa, N):
     _no_device_error(hsa)
 
 
-@pytest.mark.parametrize("N", [12032, 12033, 20000, 49152, 49153, 300001])
+@pytest.mark.parametrize("N", [12032, 12033, 20000, 49153, 75600, 360448, 360449, 500001])
 def test_partition_paths_many_and_empty_groups(hsa, N):
-    """Each of the three partition paths (rank by count up to 12032 tokens, one
-    block selecting the group boundaries up to 49152, the radix sort beyond)
-    against the oracle: 1 to 32 groups with random cuts, a run of equal values
-    straddling boundaries, and empty groups at either end."""
+    """Each of the three partition paths (rank by count up to 12032 tokens, a
+    cluster of 8 CTAs selecting the group boundaries up to 360448, the radix
+    sort beyond) against the oracle: 1 to 32 groups with random cuts, a run of
+    equal values straddling boundaries (and the CTAs' token ranges), and empty
+    groups at either end."""
     g = torch.Generator().manual_seed(N)
     stat = synth.lognormal_stat(N, 1.0, 11)
     stat[N // 3: N // 3 + 3000] = stat[7]             # ties across several boundaries
+    c = (((N + 7) // 8) + 3) & ~3                     # first token of the second CTA's range
+    stat[max(8, c - 1500): c + 1500] = stat[7]        # ties across the CTAs' ranges
     stat[5] = -0.0
     stat[6] = 0.0
     for K in (1, 2, 5, 32):
@@ -132,7 +135,7 @@ def test_partition_errors(hsa):
     bad[17] = float("-inf")
     hsa.hsa_partition(bad, 40, (40, 10), (50, 50), g, ws)
     assert hsa.hsa_get_device_error() == -5
-    for n_big in (20000, 300000):                     # the select and radix paths
+    for n_big in (20000, 300000, 400000):            # the select and radix paths
         big = torch.rand(n_big).to(DEV)
         big[n_big - 3] = float("nan")
         gb = torch.empty(n_big, dtype=torch.int32, device=DEV)
@@ -188,7 +191,7 @@ def test_active_set_workloads(hsa, name, window):
     _no_device_error(hsa)
 
 
-@pytest.mark.parametrize("N", [1, 1000, 4096, 4097, 70001, 700001])
+@pytest.mark.parametrize("N", [1, 7, 1000, 4096, 4097, 70001, 700001, 2097152, 2097153])
 def test_active_set_ragged_and_unaligned(hsa, N):
     g_ref = torch.randint(0, 3, (N,), generator=torch.Generator().manual_seed(N),
                           dtype=torch.int32)
