@@ -301,7 +301,12 @@ struct TcCfg {
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
   static constexpr int kStages = D == 128 ? 5 : 8;          // K/V ring slots
   static constexpr int kSmem = (kQT + kStages) * kTileBytes + 1024;
-  static constexpr int kOCol0 = 256;                        // O_t at kOCol0 + t*D
+  // D = 64: three S buffers in TMEM (384 columns) and O_t at 384 + 64t, so that
+  // each Q tile's next S is computed while its softmax still works on the
+  // current one.  D = 128: S_t in columns 128t, O_t at 256 + 128t.
+  static constexpr bool kThreeS = D == 64;
+  static constexpr int kOCol0 = kThreeS ? 384 : 256;        // O_t at kOCol0 + t*D
+  static constexpr int kSBars = kThreeS ? 2 : 1;            // S barriers per Q tile
 };
 
 struct TcArgs {
@@ -461,7 +466,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
   uint8_t *sQ = sm;
   uint8_t *sKV = sm + kQT * C::kTileBytes;
   __shared__ __align__(8) uint64_t bar_full[C::kStages], bar_empty[C::kStages];
-  __shared__ __align__(8) uint64_t bar_s[kQT], bar_o;
+  __shared__ __align__(8) uint64_t bar_s[kQT * C::kSBars], bar_o;
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
 
@@ -500,7 +505,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_empty[s], 1);
     }
-    for (int t = 0; t < kQT; ++t) mbar_init(&bar_s[t], 1);
+    for (int t = 0; t < kQT * C::kSBars; ++t) mbar_init(&bar_s[t], 1);
     mbar_init(&bar_o, 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -638,32 +643,80 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         named_barrier_sync(kBarP0 + t, kMeetP);
         fence_after();
       };
-      named_barrier_sync(kBarK0, 64);               // K_0 has landed
-      fence_after();
-      if (leader && !abort_flag) {
-        issue_s(0, 0);
-        mma_commit(&bar_s[0]);
-        issue_s(1, 0);
-        mma_commit(&bar_s[1]);
-      }
-      for (int j = 0; j < nT; ++j) {
-        const int Lv = 2 * j + 1, Lk = 2 * j + 2;
-        const bool more = j + 1 < nT;
-        p_ready(0);                                 // P_0(j); V_j and K_(j+1) landed
-        const bool go = leader && !abort_flag;
-        if (go) {
-          issue_o(0, Lv, j > 0);
-          if (more) {
-            issue_s(0, Lk);
-            mma_commit(&bar_s[0]);
+      if constexpr (!C::kThreeS) {
+        named_barrier_sync(kBarK0, 64);             // K_0 has landed
+        fence_after();
+        if (leader && !abort_flag) {
+          issue_s(0, 0);
+          mma_commit(&bar_s[0]);
+          issue_s(1, 0);
+          mma_commit(&bar_s[1]);
+        }
+        for (int j = 0; j < nT; ++j) {
+          const int Lv = 2 * j + 1, Lk = 2 * j + 2;
+          const bool more = j + 1 < nT;
+          p_ready(0);                               // P_0(j); V_j and K_(j+1) landed
+          const bool go = leader && !abort_flag;
+          if (go) {
+            issue_o(0, Lv, j > 0);
+            if (more) {
+              issue_s(0, Lk);
+              mma_commit(&bar_s[0]);
+            }
+          }
+          p_ready(1);
+          if (go) {
+            issue_o(1, Lv, j > 0);
+            if (more) {
+              issue_s(1, Lk);
+              mma_commit(&bar_s[1]);
+            }
           }
         }
-        p_ready(1);
-        if (go) {
-          issue_o(1, Lv, j > 0);
-          if (more) {
-            issue_s(1, Lk);
-            mma_commit(&bar_s[1]);
+      } else {
+        // Three S buffers.  The s-th S MMA in issue order (S_t(j) is number
+        // 2j + t) writes buffer s mod 3, so S_0(j+2) and S_1(j+1) reuse the
+        // buffers whose P the O MMAs just issued have read (the tensor core
+        // runs its MMAs in order).  Each Q tile's S is computed one or two key
+        // tiles ahead of its softmax.  S_t(j) completes on bar_s[2t + j%2];
+        // alternating two barriers per Q tile means no waiter can be overtaken
+        // by two completions of the barrier it waits on.
+        auto issue_s3 = [&](int t, int j) {
+          const uint64_t dq = dq0 + t * kTile16;
+          const uint64_t dk = dk0 + ((2 * j) % C::kStages) * kTile16;
+          const uint32_t ts = tmem + 128 * ((2 * j + t) % 3);
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {
+            const uint32_t off = ((k >> 2) * (kBM * 128) + (k & 3) * 32) >> 4;
+            mma_ss(ts, dq + off, dk + off, kIdS, k > 0);
+          }
+          mma_commit(&bar_s[2 * t + (j & 1)]);
+        };
+        auto issue_o3 = [&](int t, int j) {
+          const uint64_t dv = dv0 + ((2 * j + 1) % C::kStages) * kTile16;
+          const uint32_t to = tmem + C::kOCol0 + D * t, tp = tmem + 128 * ((2 * j + t) % 3);
+#pragma unroll
+          for (int k = 0; k < kBN / 16; ++k)
+            mma_ts(to, tp + 8 * k, dv + ((k * 2048) >> 4), kIdO, (j > 0 || k > 0) ? 1u : 0u);
+        };
+        named_barrier_sync(kBarK0, 64);             // K_0 (and K_1) have landed
+        fence_after();
+        if (leader && !abort_flag) {
+          issue_s3(0, 0);
+          issue_s3(1, 0);
+          if (nT > 1) issue_s3(0, 1);
+        }
+        for (int j = 0; j < nT; ++j) {
+          p_ready(0);                               // P_0(j); V_j and K_(j+1) landed
+          const bool go = leader && !abort_flag;
+          if (go) {
+            issue_o3(0, j);
+            if (j + 1 < nT) issue_s3(1, j + 1);
+          }
+          p_ready(1);                               // P_1(j); K_(j+2) landed
+          if (go) {
+            issue_o3(1, j);
+            if (j + 2 < nT) issue_s3(0, j + 2);
           }
         }
       }
@@ -697,20 +750,46 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       auto give_back = [&](int L) {
         if (lane == 0) mbar_arrive(&bar_empty[L % C::kStages]);
       };
-      landed(0);
-      named_barrier_sync(kBarK0, 64);
-      for (int j = 0; j < nT; ++j) {
-        landed(2 * j + 1);                         // V_j
-        if (j + 1 < nT) landed(2 * j + 2);         // K_(j+1)
-        named_barrier_sync(kBarP0, kMeetP);
-        if (live) {
-          live = __all_sync(0xffffffffu, mbar_wait(&bar_s[1], j & 1, &abort_flag, a.err));
+      if constexpr (!C::kThreeS) {
+        landed(0);
+        named_barrier_sync(kBarK0, 64);
+        for (int j = 0; j < nT; ++j) {
+          landed(2 * j + 1);                       // V_j
+          if (j + 1 < nT) landed(2 * j + 2);       // K_(j+1)
+          named_barrier_sync(kBarP0, kMeetP);
           if (live) {
-            give_back(2 * j);                      // K_j
-            if (j > 0) give_back(2 * j - 1);       // V_(j-1)
+            live = __all_sync(0xffffffffu, mbar_wait(&bar_s[1], j & 1, &abort_flag, a.err));
+            if (live) {
+              give_back(2 * j);                    // K_j
+              if (j > 0) give_back(2 * j - 1);     // V_(j-1)
+            }
           }
+          named_barrier_sync(kBarP0 + 1, kMeetP);
         }
-        named_barrier_sync(kBarP0 + 1, kMeetP);
+      } else {
+        // Three S buffers: K_(j+2) is needed at the meeting for P_1(j) (the
+        // issuer then issues S_0(j+2)).  S_0(j+1) is issued after O_1(j-1), so
+        // once it has completed K_j and V_(j-1) have been read by every MMA
+        // that uses them; it waits for that between the meetings for P_0(j) and
+        // P_1(j).  The next completion of the same barrier, S_0(j+3), is issued
+        // only after the meeting for P_1(j+1).
+        landed(0);                                 // K_0
+        if (nT > 1) landed(2);                     // K_1
+        named_barrier_sync(kBarK0, 64);
+        for (int j = 0; j < nT; ++j) {
+          landed(2 * j + 1);                       // V_j
+          named_barrier_sync(kBarP0, kMeetP);
+          if (live && j + 1 < nT) {
+            live = __all_sync(0xffffffffu, mbar_wait(&bar_s[(j + 1) & 1], ((j + 1) >> 1) & 1,
+                                                     &abort_flag, a.err));
+            if (live) {
+              give_back(2 * j);                    // K_j
+              if (j > 0) give_back(2 * j - 1);     // V_(j-1)
+            }
+          }
+          if (j + 2 < nT) landed(2 * j + 4);       // K_(j+2)
+          named_barrier_sync(kBarP0 + 1, kMeetP);
+        }
       }
     }
     fence_before();
@@ -739,15 +818,23 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
     // after the issuer has passed this meeting for P_t(j).
     bool ok = true;
     for (int j = 0; j < nT; ++j) {
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err));
+      if constexpr (!C::kThreeS) {
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bar_s[t], j & 1, &abort_flag, a.err));
+      } else {
+        if (ok)
+          ok = __all_sync(0xffffffffu, mbar_wait(&bar_s[2 * t + (j & 1)], (j >> 1) & 1,
+                                                 &abort_flag, a.err));
+      }
       if (ok) {
         fence_after();
         const int jg = key_tile(j);                // keys of this tile that exist
         const int valid = jg < a.tiles1 ? a.rows1 - jg * kBN : a.rows2 - (jg - a.tiles1) * kBN;
+        // three S buffers (D = 64): S_t(j) is the (2j + t)-th S MMA
+        const uint32_t tSj = C::kThreeS ? tmem + lane_off + 128 * ((2 * j + t) % 3) : tS;
         if (valid >= kBN)
-          softmax_tile<D, false>(tS, tO, valid, j == 0, sl2, m_run, l_run);
+          softmax_tile<D, false>(tSj, tO, valid, j == 0, sl2, m_run, l_run);
         else
-          softmax_tile<D, true>(tS, tO, valid, j == 0, sl2, m_run, l_run);
+          softmax_tile<D, true>(tSj, tO, valid, j == 0, sl2, m_run, l_run);
         tmem_wait_st();
       }
       fence_before();

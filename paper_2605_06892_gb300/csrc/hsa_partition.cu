@@ -280,7 +280,7 @@ cluster_select_kernel(const float *__restrict__ stat, int N, int chunk, int K, G
   cg::cluster_group cl = cg::this_cluster();
   extern __shared__ uint4 ckey4[];                     // this CTA's keys, padded to uint4
   uint32_t *skey = reinterpret_cast<uint32_t *>(ckey4);
-  __shared__ uint32_t hist[kMaxBounds * 256];          // [prefix slot][digit]
+  __shared__ __align__(16) uint32_t hist[kMaxBounds * 256];   // [prefix slot][digit]
   __shared__ uint32_t pre[kMaxBounds];                 // boundary key digits found so far
   __shared__ int below[kMaxBounds];                    // keys ordered below that prefix
   __shared__ int slot[kMaxBounds];                     // histogram of the boundary's prefix
@@ -359,13 +359,24 @@ cluster_select_kernel(const float *__restrict__ stat, int N, int chunk, int K, G
     // warp j picks boundary j's digit from the cluster's summed histogram
     if (w < nb && searched(w)) {
       const int target = gs.start[w] - below[w];       // rank among the prefix's keys
+      // bins 8*lane .. 8*lane+7 of every CTA's histogram: all 16 remote
+      // 16-byte loads are issued before they are summed
+      uint4 hv[kCsCtas][2];
+#pragma unroll
+      for (int r = 0; r < kCsCtas; ++r) {
+        const uint4 *h = reinterpret_cast<const uint4 *>(cl.map_shared_rank(hist, r) +
+                                                         slot[w] * 256 + 8 * lane);
+        hv[r][0] = h[0];
+        hv[r][1] = h[1];
+      }
       int c[8], sum = 0;
 #pragma unroll
       for (int i = 0; i < 8; ++i) c[i] = 0;
-      for (int r = 0; r < kCsCtas; ++r) {
-        const uint32_t *h = cl.map_shared_rank(hist, r) + slot[w] * 256 + 8 * lane;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) c[i] += (int)h[i];
+      for (int r = 0; r < kCsCtas; ++r) {
+        c[0] += (int)hv[r][0].x; c[1] += (int)hv[r][0].y; c[2] += (int)hv[r][0].z;
+        c[3] += (int)hv[r][0].w; c[4] += (int)hv[r][1].x; c[5] += (int)hv[r][1].y;
+        c[6] += (int)hv[r][1].z; c[7] += (int)hv[r][1].w;
       }
 #pragma unroll
       for (int i = 0; i < 8; ++i) sum += c[i];
@@ -628,12 +639,17 @@ active_set_cluster_kernel(const int32_t *__restrict__ group_of, int N, int K, ui
   for (int r = 0; r < rounds; ++r) {
     const int t = r * kAcThreads + threadIdx.x;
     const unsigned bal = bits[r * (kAcThreads / 32) + w];
-    int before = 0, total = 0;
-    for (int i = 0; i < kAcThreads / 32; ++i) {
-      const int v = __popc(bits[r * (kAcThreads / 32) + i]);
-      before += (i < w) ? v : 0;
-      total += v;
+    // active tokens of the round's earlier warps: lane i holds warp i's count,
+    // an inclusive warp scan gives every prefix
+    const int cnt = __popc(bits[r * (kAcThreads / 32) + lane]);
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
     }
+    const int before = __shfl_sync(0xffffffffu, incl - cnt, w);
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
     const int flag = (bal >> lane) & 1u;
     const int rank = base + before + __popc(bal & ((1u << lane) - 1u));
     if (t < n_loc) {
