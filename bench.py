@@ -289,6 +289,7 @@ def run_hsa(args, dist, rank, world, local_rank):
                    "l2": "flushed (256 MiB write) between steps; K/V cache and Q exceed L2",
                    "q_load": "index-driven (q_idx into the [N,H,D] query tensor)"},
         "kernels": kernels, "roofline": roofline, "dense_baseline": res["dense_baseline"],
+        "timing": res["timing"],
         "gpu_launches": res["launches"],
         "clocks": clocks,
     }
@@ -324,23 +325,23 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
 
     kinds = ("partition", "active", "gather", "scatter", "attention", "euler")
 
-    def step(record):
-        """One pass of the hot path; record(kind, fn) launches fn between events."""
+    def step(record, strm=None):
+        """One pass of the hot path; record(kind, fn) launches fn between events.
+        Launches on `strm` (default: the benchmark's stream)."""
+        st = strm if strm is not None else stream
         record("partition", lambda: hsa.hsa_partition(L.stat, T, budgets, L.counts, L.group_of,
-                                                      ws, stream))
+                                                      ws, st))
         for it in L.iters:
             n = n_of[it]
             ds = sig[it + 1] - sig[it]
             record("active", lambda: hsa.hsa_partition_active(L.group_of, T, budgets, it, L.idx,
-                                                              L.pos, w.window_pct, stream))
-            record("gather", lambda: hsa.hsa_gather_active(L.hidden, L.idx, n, L.gathered,
-                                                           stream))
+                                                              L.pos, w.window_pct, st))
+            record("gather", lambda: hsa.hsa_gather_active(L.hidden, L.idx, n, L.gathered, st))
             record("scatter", lambda: hsa.hsa_kv_sync_scatter(L.kc, L.vc, L.kf, L.vf, L.idx, n,
-                                                              stream))
+                                                              st))
             record("attention", lambda: hsa.hsa_active_attention(L.q, L.idx, n, L.kc, L.vc,
-                                                                 L.out, 0.0, ws_att, stream))
-            record("euler", lambda: hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n,
-                                                         stream))
+                                                                 L.out, 0.0, ws_att, st))
+            record("euler", lambda: hsa.hsa_cached_euler(L.x, L.vh, L.v_fresh, L.pos, ds, n, st))
 
     plain = lambda kind, fn: fn()  # noqa: E731
     for _ in range(args.warmup):
@@ -403,6 +404,7 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
             it_ms[e % n_it] += t
             if kind == "attention":
                 att_ms[e % n_it] += t
+    graph = graph_replay(args, hsa, step, plain, flush, stream, steps)
     dense = dense_iteration(args, hsa, L, sig, flush, ws_att, stream)
     by_frac = {}
     for m, it in enumerate(L.iters):
@@ -425,9 +427,42 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
         "ideal_vs_all_dense": sum(n_of.values()) / (n_it * w.N),
         "what": f"{n_it} iterations with every token active (same kernels, |A| = N), "
                 "against the measured step; L2 flushed before each dense iteration"}
+    kern_sum = sum(kern_ms.values())
+    timing = {"kernels_sum_ms": kern_sum, "gaps_ms": ms_per_step - kern_sum,
+              "graph_ms_per_step": graph,
+              "what": "kernels_sum_ms: the per-kernel CUDA-event times of a step, summed; "
+                      "gaps_ms: the rest of the step's own event time (host launch gaps "
+                      "between the event pairs); graph_ms_per_step: the same step captured "
+                      "once in a CUDA graph and replayed, L2 flushed before each replay"}
     return {"flops_step": flops_step, "ms_per_step": ms_per_step, "kernels": kernels,
             "iterations": iterations, "dense_baseline": dense_baseline, "launches": launches,
-            "clocks": clocks.summary(), "sig": sig, "n_of": n_of}
+            "clocks": clocks.summary(), "sig": sig, "n_of": n_of, "timing": timing}
+
+
+def graph_replay(args, hsa, step, plain, flush, stream, steps):
+    """The step captured once in a CUDA graph and replayed: the device time of
+    the same launches without the host's launch gaps.  The library does its host
+    work (argument checks, tensor maps, the tail plan) before enqueueing, so the
+    replay runs exactly the kernels of an eager step.  Returns ms per replay."""
+    reps = max(2, min(steps, 5))
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step(plain, torch.cuda.current_stream())     # the capture stream
+    g.replay()                                   # warm-up replay
+    torch.cuda.synchronize()
+    tot = 0.0
+    for _ in range(reps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        tot += a.elapsed_time(b)
+    assert hsa.hsa_get_device_error(stream) == 0
+    del g
+    return tot / reps
 
 
 def clock_normalised(att_tflops, clocks, peaks):
@@ -478,6 +513,7 @@ def run_also(args, hsa, dev, dist, world, local_rank, peaks):
             "partition_ms": res["kernels"]["partition"]["ms"],
             "iterations_vs_dense": {f: d["vs_dense"] for f, d in res["iterations"].items()},
             "step_vs_all_dense": res["dense_baseline"]["step_vs_all_dense"],
+            "graph_ms_per_step": res["timing"]["graph_ms_per_step"],
             "gpu_launches": res["launches"], "clocks": res["clocks"]}
         del L
         torch.cuda.empty_cache()

@@ -10,6 +10,7 @@
 // against the row count and a bad one skips its row and sets the error word.
 #include <cuda_bf16.h>
 
+#include <atomic>
 #include <cmath>
 
 #include "hsa_internal.cuh"
@@ -23,7 +24,7 @@ constexpr int kThreads = 256;
 // whose loads are contiguous, at 8; Euler holds two vectors per step).
 constexpr int kGatherUnroll = 4;
 constexpr int kScatterUnroll = 8;
-constexpr int kEulerUnroll = 4;  // float4 positions per thread per pass (large N)
+constexpr int kEulerUnroll = 2;  // float4 positions per thread per pass (large N)
 
 __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
   uint4 v;
@@ -104,11 +105,36 @@ kv_scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
 
 // x[n] = fma(vhat[n], dsigma, x[n]) with vhat[n] refreshed from
 // v_fresh[pos[n]] when pos[n] >= 0.  Element-wise over the N*C/4 float4
-// vectors: each thread takes kEulerUnroll vectors a grid-stride apart, loads
-// their pos entries, then all their x and velocity vectors, then stores, so
-// 3*kEulerUnroll independent loads are in flight per thread whatever C is.
+// vectors: each thread takes kU vectors a grid-stride apart.  The pos entries
+// of a pass are loaded one pass ahead (software pipelining), so a pass issues
+// its x loads and its velocity loads (v_fresh rows by pos, or the cache)
+// at once: 2*kU independent loads in flight per thread whatever C is.  The
+// grid is the number of blocks resident at once (a single wave).  Measured on
+// GB300 with an L2-flushed size sweep: kU = 2 with the pos loads one pass
+// ahead reaches 0.85-1.0 of the HBM copy rate, kU = 4 (more registers, fewer
+// resident threads) 0.68-0.85.
 // vec_shift = log2(C/4) when C/4 is a power of two, else -1 (division).
 // Small N uses one vector per thread (kU = 1) so that every SM has work.
+template <int kU>
+__device__ __forceinline__ void load_pos_pass(const int32_t *__restrict__ pos, long long base,
+                                              long long stride, long long total, int vecs,
+                                              int vec_shift, int n_fresh_rows, unsigned *err,
+                                              int (&p)[kU]) {
+#pragma unroll
+  for (int u = 0; u < kU; ++u) {
+    const long long e = base + u * stride;
+    p[u] = -1;
+    if (pos && e < total) {
+      const long long row = vec_shift >= 0 ? (e >> vec_shift) : e / vecs;
+      p[u] = __ldg(pos + row);
+      if (p[u] >= n_fresh_rows || p[u] < -1) {   // only -1 means "no fresh row"
+        set_error(err, kErrIndex);
+        p[u] = -1;
+      }
+    }
+  }
+}
+
 template <int kU>
 __global__ void __launch_bounds__(kThreads)
 cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
@@ -116,42 +142,106 @@ cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
                     long long total, int vecs, int vec_shift, float dsigma, int n_fresh_rows,
                     unsigned *err) {
   const long long stride = (long long)gridDim.x * blockDim.x;
-  for (long long base = blockIdx.x * (long long)blockDim.x + threadIdx.x; base < total;
-       base += stride * kU) {
-    long long e[kU], row[kU];
+  long long base = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  int pn[kU];
+  load_pos_pass<kU>(pos, base, stride, total, vecs, vec_shift, n_fresh_rows, err, pn);
+  for (; base < total; base += stride * kU) {
     int p[kU];
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      e[u] = base + u * stride;
-      row[u] = vec_shift >= 0 ? (e[u] >> vec_shift) : e[u] / vecs;
-      p[u] = -1;
-      if (pos && e[u] < total) {
-        p[u] = __ldg(pos + row[u]);
-        if (p[u] >= n_fresh_rows || p[u] < -1) {   // only -1 means "no fresh row"
-          set_error(err, kErrIndex);
-          p[u] = -1;
-        }
-      }
-    }
+    for (int u = 0; u < kU; ++u) p[u] = pn[u];
+    load_pos_pass<kU>(pos, base + stride * kU, stride, total, vecs, vec_shift, n_fresh_rows,
+                      err, pn);
     float4 vb[kU], xb[kU];
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      if (e[u] < total) {
-        const long long c = e[u] - row[u] * vecs;
-        vb[u] = p[u] >= 0 ? __ldg(v_fresh + (long long)p[u] * vecs + c) : vhat[e[u]];
-        xb[u] = x[e[u]];
+      const long long e = base + u * stride;
+      if (e < total) {
+        const long long row = vec_shift >= 0 ? (e >> vec_shift) : e / vecs;
+        const long long c = e - row * vecs;
+        xb[u] = x[e];
+        vb[u] = p[u] >= 0 ? __ldg(v_fresh + (long long)p[u] * vecs + c) : vhat[e];
       }
     }
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      if (e[u] < total) {
-        if (p[u] >= 0) vhat[e[u]] = vb[u];
+      const long long e = base + u * stride;
+      if (e < total) {
+        if (p[u] >= 0) vhat[e] = vb[u];
         float4 o;
         o.x = __fmaf_rn(vb[u].x, dsigma, xb[u].x);
         o.y = __fmaf_rn(vb[u].y, dsigma, xb[u].y);
         o.z = __fmaf_rn(vb[u].z, dsigma, xb[u].z);
         o.w = __fmaf_rn(vb[u].w, dsigma, xb[u].w);
-        x[e[u]] = o;
+        x[e] = o;
+      }
+    }
+  }
+}
+
+// The cached Euler step fused with the velocity statistic (below), element-
+// wise like cached_euler_kernel, for C/4 a power of two <= 32: the C/4 lanes
+// of a token are consecutive lanes of one warp (passes start at a multiple of
+// 32), so the token's two L1 norms are reduced with log2(C/4) shuffles and the
+// token's first lane updates stat.  Every lane of a warp runs the same passes
+// (the shuffles span the warp).
+template <int kU>
+__global__ void __launch_bounds__(kThreads)
+euler_l1rel_elem_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
+                        const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
+                        long long total, int vecs, int vec_shift, float dsigma,
+                        int n_fresh_rows, float *__restrict__ stat, float weight, unsigned *err) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  long long base = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  int pn[kU];
+  load_pos_pass<kU>(pos, base, stride, total, vecs, vec_shift, n_fresh_rows, err, pn);
+  for (; base - lane < total; base += stride * kU) {
+    int p[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) p[u] = pn[u];
+    load_pos_pass<kU>(pos, base + stride * kU, stride, total, vecs, vec_shift, n_fresh_rows,
+                      err, pn);
+    float4 vo[kU], vn[kU], xb[kU];
+    float st[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const long long e = base + u * stride;
+      st[u] = 0.f;
+      if (e < total) {
+        const long long row = e >> vec_shift;
+        const long long c = e - row * vecs;
+        xb[u] = x[e];
+        vo[u] = vhat[e];
+        vn[u] = p[u] >= 0 ? __ldg(v_fresh + (long long)p[u] * vecs + c) : vo[u];
+        if (p[u] >= 0 && (lane & (vecs - 1)) == 0) st[u] = stat[row];   // with the data
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const long long e = base + u * stride;
+      float num = 0.f, den = 0.f;
+      if (e < total) {
+        if (p[u] >= 0) {
+          num = fabsf(vn[u].x - vo[u].x) + fabsf(vn[u].y - vo[u].y) + fabsf(vn[u].z - vo[u].z) +
+                fabsf(vn[u].w - vo[u].w);
+          den = fabsf(vn[u].x) + fabsf(vn[u].y) + fabsf(vn[u].z) + fabsf(vn[u].w);
+          vhat[e] = vn[u];
+        }
+        float4 o;
+        o.x = __fmaf_rn(vn[u].x, dsigma, xb[u].x);
+        o.y = __fmaf_rn(vn[u].y, dsigma, xb[u].y);
+        o.z = __fmaf_rn(vn[u].z, dsigma, xb[u].z);
+        o.w = __fmaf_rn(vn[u].w, dsigma, xb[u].w);
+        x[e] = o;
+      }
+      for (int o = 1; o < vecs; o <<= 1) {
+        num += __shfl_xor_sync(0xffffffffu, num, o);
+        den += __shfl_xor_sync(0xffffffffu, den, o);
+      }
+      if (e < total && p[u] >= 0 && (lane & (vecs - 1)) == 0) {
+        const long long row = e >> vec_shift;
+        const float r = den > 0.f ? num / den : (num > 0.f ? 3.402823466e38f : 0.f);
+        stat[row] = fmaf(weight, r, st[u]);
       }
     }
   }
@@ -162,8 +252,9 @@ cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
 // row is v_{i-1}[n] and the fresh row v_i[n]; the kernel adds
 // weight * ||v_i - v_{i-1}||_1 / ||v_i||_1 to stat[n] (a zero denominator
 // counts 0 with a zero numerator, FLT_MAX otherwise), then refreshes the cache
-// and advances x exactly as cached_euler_kernel does.  A group of L lanes owns
-// a token; the two L1 norms are reduced across the group with shuffles.
+// and advances x exactly as cached_euler_kernel does.  This layout (for C/4
+// not a power of two, or above 32): a group of L lanes owns a token; the two
+// L1 norms are reduced across the group with shuffles.
 constexpr int kL1relRows = 2;   // tokens per lane group per pass
 
 __global__ void __launch_bounds__(kThreads, 4)
@@ -374,6 +465,24 @@ int grid_for(long long n_rows, int L) {
   return (int)(blocks < 1 ? 1 : blocks);
 }
 
+// Blocks of kernel K (kThreads threads) resident on the whole device at once,
+// resolved once per device: a grid-stride kernel launched with this many
+// blocks runs in a single wave.
+template <auto K>
+long long resident_blocks() {
+  static std::atomic<int> per_sm[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return sm_count();
+  int nb = per_sm[dev].load(std::memory_order_relaxed);
+  if (nb <= 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, K, kThreads, 0) != cudaSuccess ||
+        nb < 1)
+      nb = 1;
+    per_sm[dev].store(nb, std::memory_order_relaxed);
+  }
+  return (long long)nb * sm_count();
+}
+
 int log2i(int L) {
   int s = 0;
   while ((1 << s) < L) ++s;
@@ -444,7 +553,8 @@ extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
   const long long resident = (long long)sm_count() * 2048;     // threads
   const int per = total >= (long long)kEulerUnroll * resident ? kEulerUnroll : 1;
   long long blocks = (total + (long long)kThreads * per - 1) / ((long long)kThreads * per);
-  const long long cap = (long long)sm_count() * (2048 / kThreads);
+  const long long cap = per == kEulerUnroll ? resident_blocks<cached_euler_kernel<kEulerUnroll>>()
+                                            : resident_blocks<cached_euler_kernel<1>>();
   if (blocks > cap) blocks = cap;
   count_launches(1);
   if (per == kEulerUnroll)
@@ -470,6 +580,30 @@ extern "C" int hsa_cached_euler_l1rel(float *x, float *v_cache, const float *v_f
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
   const int vecs = C / 4;
+  int vec_shift = -1;
+  for (int sh = 0; sh <= 5; ++sh)
+    if ((1 << sh) == vecs) vec_shift = sh;
+  if (vec_shift >= 0) {
+    // element-wise: C/4 a power of two, at most 32 (a token within one warp)
+    const long long total = (long long)N * vecs;
+    const long long resident = (long long)sm_count() * 2048;     // threads
+    const int per = total >= (long long)kEulerUnroll * resident ? kEulerUnroll : 1;
+    long long blocks = (total + (long long)kThreads * per - 1) / ((long long)kThreads * per);
+    const long long cap = per == kEulerUnroll
+                              ? resident_blocks<euler_l1rel_elem_kernel<kEulerUnroll>>()
+                              : resident_blocks<euler_l1rel_elem_kernel<1>>();
+    if (blocks > cap) blocks = cap;
+    count_launches(1);
+    if (per == kEulerUnroll)
+      euler_l1rel_elem_kernel<kEulerUnroll><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
+          (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
+          dsigma, n_fresh, stat, weight, err);
+    else
+      euler_l1rel_elem_kernel<1><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
+          (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
+          dsigma, n_fresh, stat, weight, err);
+    return launch_status();
+  }
   const int L = lanes_per_row(vecs);
   count_launches(1);
   euler_l1rel_kernel<<<grid_for(((long long)N + kL1relRows - 1) / kL1relRows, L), kThreads, 0,
