@@ -541,13 +541,19 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
       if (i < kVecs && grow < a.n_active) src[u] = a.q_idx ? __ldg(a.q_idx + grow) : grow;
     }
     uint4 v[kPer];
+    uint64_t pol;                       // the query rows are read once: evict first
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
       const int i = threadIdx.x + u * kTcThreads;
       v[u] = make_uint4(0u, 0u, 0u, 0u);
-      if (src[u] >= 0 && src[u] < a.q_rows)
-        v[u] = __ldg(reinterpret_cast<const uint4 *>(a.q + (size_t)src[u] * row_stride +
-                                                     (size_t)h * D) + i % kVecPerRow);
+      if (src[u] >= 0 && src[u] < a.q_rows) {
+        const uint4 *p = reinterpret_cast<const uint4 *>(a.q + (size_t)src[u] * row_stride +
+                                                         (size_t)h * D) + i % kVecPerRow;
+        asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
+                     : "=r"(v[u].x), "=r"(v[u].y), "=r"(v[u].z), "=r"(v[u].w)
+                     : "l"(p), "l"(pol));
+      }
       else if (i < kVecs && row0 + i / kVecPerRow < a.n_active && i % kVecPerRow == 0)
         set_error(a.err, kErrIndex);
     }
@@ -873,10 +879,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         for (int i = 0; i < 16; ++i)
           pk[i] = pack_bf16(__uint_as_float(o[2 * i]) * inv, __uint_as_float(o[2 * i + 1]) * inv);
         if (grow < a.n_active) {
-          uint4 *d4 = reinterpret_cast<uint4 *>(dst + 32 * c);
+          uint64_t pol;                 // the output rows are written once: evict first
+          asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
 #pragma unroll
           for (int v = 0; v < 4; ++v)
-            d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+            asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1,%2,%3,%4}, %5;" ::"l"(
+                             dst + 32 * c + 8 * v),
+                         "r"(pk[4 * v]), "r"(pk[4 * v + 1]), "r"(pk[4 * v + 2]),
+                         "r"(pk[4 * v + 3]), "l"(pol)
+                         : "memory");
         }
       }
     }
