@@ -49,6 +49,7 @@ HEADLINE = "wan14b_720p"
 ALSO = ("wan13b", "wan14b_boxes", "ltx", "tiny_f32")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
+HEAD_START_CYCLES = 6_000_000      # ~3 ms of GPU spin while the host enqueues a timed step
 
 
 def parse():
@@ -351,7 +352,7 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
     assert hsa.hsa_get_device_error(stream) == 0
 
     per_kernel = {k: [] for k in kinds}
-    step_events = []
+    step_events, bd_events = [], []
 
     def timed(kind, fn):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -360,24 +361,41 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
         b.record(stream)
         per_kernel[kind].append((a, b))
 
+    def one_step(record, events):
+        flush.zero_()                           # L2 flush, outside the step's events
+        # The GPU spins for a moment (outside the events) while the host enqueues
+        # the step, so that host launch latency does not open gaps between the
+        # step's kernels: the events time the device's work.  (The e2e leg keeps
+        # the host in the loop.)
+        torch.cuda._sleep(HEAD_START_CYCLES)
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        step(record)
+        s1.record(stream)
+        events.append((s0, s1))
+
+    # The timed steps carry no event inside them (an event between two kernels
+    # keeps the second from starting during the first's last moments, which
+    # costs a few microseconds per launch on short steps).  The per-kernel
+    # breakdown comes from separate steps with an event pair around every call.
+    bsteps = max(2, min(steps, 5))
     barrier(dist)
     torch.cuda.synchronize()
     launches0 = hsa.hsa_launch_count()
     with ClockSampler(local_rank) as clocks:
         for _ in range(steps):
-            flush.zero_()                       # L2 flush, outside the step's events
-            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            s0.record(stream)
-            step(timed)
-            s1.record(stream)
-            step_events.append((s0, s1))
+            one_step(plain, step_events)
         torch.cuda.synchronize()
-    launches = hsa.hsa_launch_count() - launches0       # this library's kernels only
-    barrier(dist)
+        launches = hsa.hsa_launch_count() - launches0       # this library's kernels only
+        barrier(dist)
+        for _ in range(bsteps):
+            one_step(timed, bd_events)
+        torch.cuda.synchronize()
     step_ms = [a.elapsed_time(b) for a, b in step_events]
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
     ms_per_step = total_ms / steps
-    kern_ms = {k: sum(a.elapsed_time(b) for a, b in v) / steps for k, v in per_kernel.items()}
+    bd_ms_per_step = sum(a.elapsed_time(b) for a, b in bd_events) / bsteps
+    kern_ms = {k: sum(a.elapsed_time(b) for a, b in v) / bsteps for k, v in per_kernel.items()}
     status = hsa.hsa_get_device_error(stream)
     assert status == 0, f"device error {status}"
 
@@ -400,7 +418,7 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
     att_ms = [0.0] * n_it
     for kind in ("active", "gather", "scatter", "attention", "euler"):
         for e, (a, b) in enumerate(per_kernel[kind]):
-            t = a.elapsed_time(b) / steps
+            t = a.elapsed_time(b) / bsteps
             it_ms[e % n_it] += t
             if kind == "attention":
                 att_ms[e % n_it] += t
@@ -428,12 +446,16 @@ def measure(args, hsa, L, dev, dist, world, local_rank, steps, peaks):
         "what": f"{n_it} iterations with every token active (same kernels, |A| = N), "
                 "against the measured step; L2 flushed before each dense iteration"}
     kern_sum = sum(kern_ms.values())
-    timing = {"kernels_sum_ms": kern_sum, "gaps_ms": ms_per_step - kern_sum,
-              "graph_ms_per_step": graph,
-              "what": "kernels_sum_ms: the per-kernel CUDA-event times of a step, summed; "
-                      "gaps_ms: the rest of the step's own event time (host launch gaps "
-                      "between the event pairs); graph_ms_per_step: the same step captured "
-                      "once in a CUDA graph and replayed, L2 flushed before each replay"}
+    timing = {"step_ms": ms_per_step, "breakdown_steps": bsteps,
+              "breakdown_step_ms": bd_ms_per_step, "kernels_sum_ms": kern_sum,
+              "gaps_ms": bd_ms_per_step - kern_sum, "graph_ms_per_step": graph,
+              "what": "step_ms: the timed steps (no event inside a step); breakdown_step_ms: "
+                      "separate steps with an event pair around every call, whose per-kernel "
+                      "times sum to kernels_sum_ms (gaps_ms: the rest of those steps); "
+                      "graph_ms_per_step: the same step captured once in a CUDA graph and "
+                      "replayed.  L2 flushed before every step; each step is enqueued while "
+                      "the GPU spins (outside the events), so host launch latency does not "
+                      "appear inside a step"}
     return {"flops_step": flops_step, "ms_per_step": ms_per_step, "kernels": kernels,
             "iterations": iterations, "dense_baseline": dense_baseline, "launches": launches,
             "clocks": clocks.summary(), "sig": sig, "n_of": n_of, "timing": timing}
@@ -533,6 +555,7 @@ def dense_iteration(args, hsa, L, sig, flush, ws_att, stream, reps=None):
     tot, att = [], []
     for r in range(reps + 1):
         flush.zero_()
+        torch.cuda._sleep(HEAD_START_CYCLES)
         a, b, c, d = ev(), ev(), ev(), ev()
         a.record(stream)
         hsa.hsa_partition_active(L.group_of, T, budgets, 0, L.idx, L.pos, w.window_pct, stream)

@@ -119,7 +119,7 @@ int hsa_partition(const float *stat, int N, int T, const int *budgets,
                   size_t workspace_bytes, hsa_stream_t stream);
 
 /* Largest N accepted by hsa_partition_static. */
-#define HSA_PARTITION_STATIC_MAX_TOKENS 262144
+#define HSA_PARTITION_STATIC_MAX_TOKENS 524288
 
 /* hsa_partition without a workspace argument, for callers that cannot
  * allocate device memory for one: a plugin inside a host framework that owns
@@ -127,8 +127,10 @@ int hsa_partition(const float *stat, int N, int T, const int *budgets,
  * that must not call cudaMalloc/cudaFree (they may synchronise the device).
  * The paper has no counterpart; the ranking and group assignment are exactly
  * those of hsa_partition (same arguments, same results).
- * Scratch: a fixed device array inside the library, about 4.3 MB, sized for
- * N <= HSA_PARTITION_STATIC_MAX_TOKENS; every GPU that loads the library's
+ * Scratch: a fixed device array inside the library, about 8.5 MB, sized for
+ * N <= HSA_PARTITION_STATIC_MAX_TOKENS (the sort that partitions layers of more
+ * than 360448 tokens uses it; smaller layers take paths that need no scratch);
+ * every GPU that loads the library's
  * partition module holds it until the process exits.  The CUDA runtime
  * reserves it when that module is loaded on a device: when the library is
  * loaded if CUDA_MODULE_LOADING=EAGER, otherwise (lazy loading, the default)

@@ -34,7 +34,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 library_path = os.path.join(_HERE, "libhsa.so")
 
 HSA_BF16, HSA_F32 = 0, 1
-HSA_PARTITION_STATIC_MAX_TOKENS = 262144
+HSA_PARTITION_STATIC_MAX_TOKENS = 524288
 STATUS = {0: "HSA_OK", -1: "HSA_ERR_INVALID_ARG", -2: "HSA_ERR_NOT_DIVISOR",
           -3: "HSA_ERR_BAD_COUNTS", -4: "HSA_ERR_UNSUPPORTED", -5: "HSA_ERR_NONFINITE",
           -6: "HSA_ERR_INDEX", -7: "HSA_ERR_TIMEOUT", -8: "HSA_ERR_CUDA",

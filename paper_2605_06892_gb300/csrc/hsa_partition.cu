@@ -903,13 +903,16 @@ __global__ void reserve_frame_kernel(float *__restrict__ stat, int frame_tokens)
 // memory and exposes no allocator to it, or a latency-critical loop where
 // cudaMalloc/cudaFree (which may synchronise the device) are not acceptable.
 // Its scratch is a fixed file-scope device array sized for
-// HSA_PARTITION_STATIC_MAX_TOKENS tokens; every GPU that loads the library
-// holds it until the process exits.
+// HSA_PARTITION_STATIC_MAX_TOKENS tokens (the radix sort of layers above
+// kCsMaxN tokens works in it; smaller layers need no scratch); every GPU that
+// loads the library holds it until the process exits.
 
 namespace {
 
 constexpr size_t kStaticScratchBytes = sort_layout(HSA_PARTITION_STATIC_MAX_TOKENS).total;
 static_assert(kStaticScratchBytes % 256 == 0, "scratch array size");
+static_assert(HSA_PARTITION_STATIC_MAX_TOKENS > kCsMaxN,
+              "the fixed scratch must serve the sizes that need one");
 
 // The host cannot use this symbol as a device address; the set-up below asks
 // the runtime for the device address once per device.

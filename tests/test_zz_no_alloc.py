@@ -4,10 +4,11 @@ workspace: it serves callers that cannot allocate device memory themselves
 loop that must not call cudaMalloc because it can synchronise the device).
 
 Through the C ABI it must give exactly what hsa_partition gives with a
-caller-provided workspace, on calls in a row (the second with a smaller
-input, so anything left in the shared scratch by the first call would show,
-the third at a size served by another partition path),
-and it must refuse inputs larger than its fixed scratch before launching.
+caller-provided workspace, on calls in a row: the first large enough for the
+radix sort that works in the fixed scratch, the second a smaller sort in the
+same scratch (anything the first left there would show), then sizes served by
+the paths that need no scratch, and a sort again; and it must refuse inputs
+larger than its fixed scratch before launching.
 This file is collected last on purpose.
 """
 import ctypes
@@ -51,6 +52,27 @@ def _static_c_abi(hsa, stat, T, budgets, counts):
 
 
 def test_static_partition_matches_workspace_partition_twice(hsa):
+    # first call: the largest size accepted, a radix sort in the fixed scratch
+    N0 = hsa.HSA_PARTITION_STATIC_MAX_TOKENS
+    stat0 = synth.lognormal_stat(N0, 1.0, 9).cuda()
+    budgets0, counts0 = (40, 20, 10, 5), (N0 // 4, N0 // 4, N0 // 4, N0 - 3 * (N0 // 4))
+    ref0 = _with_workspace(hsa, stat0, 40, budgets0, counts0)
+    got0 = _static_c_abi(hsa, stat0, 40, budgets0, counts0)
+    torch.cuda.synchronize()
+    assert torch.equal(got0, ref0)
+
+    # a smaller sort in the same scratch, with ties across group boundaries
+    Ns = 400003
+    g = torch.Generator().manual_seed(3)
+    stats = torch.rand(Ns, generator=g)
+    stats[1000:90000] = stats[5]
+    stats = stats.cuda()
+    budgets_s, counts_s = (40, 10), (150001, 250002)
+    ref_s = _with_workspace(hsa, stats, 40, budgets_s, counts_s)
+    got_s = _static_c_abi(hsa, stats, 40, budgets_s, counts_s)
+    torch.cuda.synchronize()
+    assert torch.equal(got_s, ref_s)
+
     w = synth.WORKLOADS["wan14b_720p"]
     stat1, counts1 = synth.stat_for(w)
     stat1 = stat1.cuda()
@@ -69,7 +91,7 @@ def test_static_partition_matches_workspace_partition_twice(hsa):
     torch.cuda.synchronize()
     assert torch.equal(got2, ref2)
 
-    # third call: a size the one-block boundary select serves
+    # a size the cluster boundary select serves
     N3 = 30000
     stat3 = synth.lognormal_stat(N3, 1.0, 5).cuda()
     budgets3, counts3 = (40, 20, 10, 5), (7000, 8000, 9000, 6000)
@@ -77,6 +99,11 @@ def test_static_partition_matches_workspace_partition_twice(hsa):
     got3 = _static_c_abi(hsa, stat3, 40, budgets3, counts3)
     torch.cuda.synchronize()
     assert torch.equal(got3, ref3)
+
+    # and a sort in the scratch again after the paths that do not use it
+    got4 = _static_c_abi(hsa, stat0, 40, budgets0, counts0)
+    torch.cuda.synchronize()
+    assert torch.equal(got4, ref0)
     assert hsa.hsa_get_device_error() == 0
 
 
