@@ -22,10 +22,15 @@
 //               the S columns, and at the end normalises O and stores it.
 //   all warps   load the 256 query rows once, by index, into swizzled smem.
 // The two Q tiles ping-pong: while one softmax group works on its scores the
-// tensor core runs the other tile's MMAs.  The issuer waits only on hardware
+// tensor core runs the other tile's MMAs.  At D = 64 the TMEM also has room for
+// a third S buffer, so each Q tile's next scores are computed while its softmax
+// still works on the current ones.  The issuer waits only on hardware
 // named barriers, two per key tile (P of a tile, with the K/V tiles the next
 // MMAs read), where the other roles meet it; an mbarrier test on its path
-// would idle the tensor core.  After the
+// would idle the tensor core.  Units of odd waves walk their keys backwards
+// (so they start on the tiles the previous wave of the head read last, still
+// in L2), and the query and output rows, read and written once, are marked
+// for early L2 eviction.  After the
 // first key tile the probabilities are formed against the running reference
 // maximum without computing the tile's maximum; only if a row sum would pass
 // 2^32 is the tile redone with its exact maximum (and O rescaled in TMEM).

@@ -695,6 +695,30 @@ bool cluster_select_ready() {
   return st == 1;
 }
 
+// The same check for the active-set cluster (8 CTAs of 1024 threads, 33 KB of
+// static shared memory each); otherwise the active set takes the per-block
+// scheme.
+bool cluster_active_ready() {
+  static std::atomic<int> state[64];            // 0 unknown, 1 ready, 2 unavailable
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  int st = state[dev].load();
+  if (st == 0) {
+    st = 2;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kCsCtas);
+    cfg.blockDim = dim3(kAcThreads);
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, active_set_cluster_kernel, &cfg) ==
+            cudaSuccess &&
+        clusters >= 1)
+      st = 1;
+    cudaGetLastError();                          // a refused query leaves no sticky error
+    state[dev].store(st);
+  }
+  return st == 1;
+}
+
 }  // namespace
 
 extern "C" size_t hsa_partition_workspace_bytes(int N) {
@@ -781,7 +805,7 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
   cudaStream_t s = (cudaStream_t)stream;
   unsigned *err = device_error_word();
   if (!err) return HSA_ERR_CUDA;
-  if (N <= kAcMaxN) {
+  if (N <= kAcMaxN && cluster_active_ready()) {
     const int chunk = (N + kCsCtas - 1) / kCsCtas;
     count_launches(1);
     active_set_cluster_kernel<<<kCsCtas, kAcThreads, 0, s>>>(group_of, N, K, mask, chunk, idx,
