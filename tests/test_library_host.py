@@ -109,3 +109,39 @@ def test_launch_counter_needs_no_gpu(hsa):
     st = hsa.lib().hsa_partition(None, 4, 40, ints(40, 15), ints(2, 2), 2, None, None, 0, None)
     assert st < 0
     assert hsa.hsa_launch_count() == c0
+
+
+def test_index_check_host_side(hsa):
+    """hsa_check_indices: one bit per token of workspace, in whole 256-byte
+    blocks; argument and workspace errors are reported on the host before any
+    launch (so no GPU is needed to see them)."""
+    ws = hsa.lib().hsa_check_indices_workspace_bytes
+    assert ws(0) == 0
+    for N in (1, 31, 32, 2048, 2049, 75600, 10 ** 6):
+        b = ws(N)
+        assert b % 256 == 0 and b * 8 >= N and b - 256 < (N + 7) // 8 + 16
+    c0 = hsa.hsa_launch_count()
+    lib = hsa.lib()
+    assert lib.hsa_check_indices(None, 0, 100, None, 0, None) == 0          # nothing to check
+    assert lib.hsa_check_indices(None, -1, 100, None, 0, None) == -1        # n < 0
+    assert lib.hsa_check_indices(None, 5, 100, None, 0, None) == -1        # no idx
+    fake = ctypes.c_void_p(4096)                                           # never dereferenced
+    assert lib.hsa_check_indices(fake, 5, 100, None, 0, None) == -9        # no workspace
+    assert lib.hsa_check_indices(fake, 5, 10 ** 6, fake, 256, None) == -9  # too small
+    assert lib.hsa_check_indices(fake, 5, 100, ctypes.c_void_p(4100), 256, None) == -9  # misaligned
+    assert hsa.hsa_launch_count() == c0
+
+
+def test_static_partition_limit_agrees(hsa):
+    """The binding's copy of HSA_PARTITION_STATIC_MAX_TOKENS is the header's, and
+    the limit lies above the sizes that the partition serves without scratch
+    (the cluster select ends at 360448 tokens), so the fixed array is used."""
+    src = open(os.path.join(ROOT, "include", "hsa.h")).read()
+    m = re.search(r"#define\s+HSA_PARTITION_STATIC_MAX_TOKENS\s+(\d+)", src)
+    assert m and int(m.group(1)) == hsa.HSA_PARTITION_STATIC_MAX_TOKENS
+    assert hsa.HSA_PARTITION_STATIC_MAX_TOKENS > 360448
+    ints = ctypes.c_int * 1
+    st = hsa.lib().hsa_partition_static(None, hsa.HSA_PARTITION_STATIC_MAX_TOKENS + 1, 8,
+                                        ints(8), ints(hsa.HSA_PARTITION_STATIC_MAX_TOKENS + 1),
+                                        1, None, None)
+    assert st == -4                                                        # before any launch
