@@ -393,14 +393,16 @@ __device__ __forceinline__ float exp_store_tile(uint32_t tS, const uint32_t (&r)
 // after the first tile P is formed against m_run without looking at this
 // tile's maximum (fast path).  If a row's sum then exceeds 2^32 (or is not
 // finite) the warp redoes the tile on the exact path: the row maximum of the
-// scores (still in registers) becomes the new reference, O (in TMEM, idle
-// now: this tile's S is complete, so the previous O += P V is too) and the
-// running sum take the factor 2^(m_old - m_new), and P is formed again.  The
-// first tile always takes the exact path.  kTail masks keys >= valid (the
-// last, ragged tile); full tiles take no per-key test.
-template <int D, bool kTail>
+// scores (still in registers) becomes the new reference, O (in TMEM) and the
+// running sum take the factor 2^(m_old - m_new), and P is formed again.  O is
+// rescaled only once o_idle() has returned true: the previous O += P V has
+// then completed (false: a wait failed, O is left alone).  The first tile
+// always takes the exact path.  kTail masks keys >= valid (the last, ragged
+// tile); full tiles take no per-key test.
+template <int D, bool kTail, typename OIdle>
 __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid, bool first,
-                                             float sl2, float &m_run, float &l_run) {
+                                             float sl2, float &m_run, float &l_run,
+                                             OIdle &&o_idle) {
   // The second half of S is read while the first half is masked.
   uint32_t r[128];
   tmem_ld32(tS, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
@@ -445,7 +447,7 @@ __device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int valid
   const float alpha = (!first && m_new > m_run) ? fast_exp2(m_run - m_new) : 1.f;
   l_run = first ? 0.f : l_run * alpha;
   m_run = m_new;
-  if (!first && __any_sync(0xffffffffu, alpha != 1.f)) {
+  if (!first && __any_sync(0xffffffffu, alpha != 1.f) && o_idle()) {
 #pragma unroll
     for (int c = 0; c < D / 16; ++c) {
       uint32_t o[16];
@@ -727,7 +729,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
           p_ready(1);                               // P_1(j); K_(j+2) landed
           if (go) {
             issue_o3(1, j);
-            if (j + 2 < nT) issue_s3(0, j + 2);
+            if (j + 2 < nT)
+              issue_s3(0, j + 2);
+            else if (j + 2 == nT)
+              mma_commit(&bar_s[(j + 2) & 1]);      // O_1(j) done, for the last tile's rescale
           }
         }
       }
@@ -842,10 +847,24 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__
         const int valid = jg < a.tiles1 ? a.rows1 - jg * kBN : a.rows2 - (jg - a.tiles1) * kBN;
         // three S buffers (D = 64): S_t(j) is the (2j + t)-th S MMA
         const uint32_t tSj = C::kThreeS ? tmem + lane_off + 128 * ((2 * j + t) % 3) : tS;
+        // O_t(j-1) has completed once an MMA issued after it has.  With two
+        // S buffers that is S_t(j), complete already.  With three, S_t(j) is
+        // issued before O_t(j-1): wait for S_1(j) (Q tile 0) or S_0(j+1) (Q
+        // tile 1; at the last key tile the issuer commits that barrier with
+        // no MMA).  Neither barrier can complete again before this warp's
+        // next meeting.  Needed only on the exact path's rescale, so rare.
+        auto o_idle = [&]() -> bool {
+          if constexpr (!C::kThreeS) return true;
+          uint64_t *b = t == 0 ? &bar_s[2 + (j & 1)] : &bar_s[(j + 1) & 1];
+          const uint32_t par = t == 0 ? (j >> 1) & 1 : ((j + 1) >> 1) & 1;
+          const bool idle = __all_sync(0xffffffffu, mbar_wait(b, par, &abort_flag, a.err));
+          fence_after();
+          return idle;
+        };
         if (valid >= kBN)
-          softmax_tile<D, false>(tSj, tO, valid, j == 0, sl2, m_run, l_run);
+          softmax_tile<D, false>(tSj, tO, valid, j == 0, sl2, m_run, l_run, o_idle);
         else
-          softmax_tile<D, true>(tSj, tO, valid, j == 0, sl2, m_run, l_run);
+          softmax_tile<D, true>(tSj, tO, valid, j == 0, sl2, m_run, l_run, o_idle);
         tmem_wait_st();
       }
       fence_before();
