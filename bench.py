@@ -260,19 +260,6 @@ def run_hsa(args, dist, rank, world, local_rank):
     L = Layer(w, dev, keep_host=want_cpu)
     peaks, peak_src = load_peaks()
     res = measure(args, hsa, L, dev, dist, world, local_rank, args.steps, peaks)
-    also = {}
-    with_also = (not args.no_also and not args.heads and not args.iters
-                 and args.workload == HEADLINE)
-    if with_also:
-        # The same layer and inputs with the HSA-50 preset's caching window
-        # (k = 80 %: the first and last m = 4 iterations are full passes).
-        wk = dataclasses.replace(w, name=w.name + "_window80", window_pct=80)
-        L.w = wk
-        steps = max(3, min(args.steps, 10))
-        also[wk.name] = also_summary(
-            wk, L.counts, steps, measure(args, hsa, L, dev, dist, world, local_rank, steps,
-                                         peaks), peaks, world)
-        L.w = w
     flops_step, ms_per_step = res["flops_step"], res["ms_per_step"]
     value = world * flops_step / (ms_per_step * 1e-3) / 1e12
     kernels = res["kernels"]
@@ -312,6 +299,18 @@ def run_hsa(args, dist, rank, world, local_rank):
                               dev, dist, world, flops_step, local_rank)
     if want_cpu:
         line["cpu_baseline"] = cpu_baseline(w, L)
+    with_also = (not args.no_also and not args.heads and not args.iters
+                 and args.workload == HEADLINE)
+    also = {}
+    if with_also:
+        # The same layer and inputs with the HSA-50 preset's caching window
+        # (k = 80 %: the first and last m = 4 iterations are full passes).
+        wk = dataclasses.replace(w, name=w.name + "_window80", window_pct=80)
+        L.w = wk
+        steps = max(3, min(args.steps, 10))
+        also[wk.name] = also_summary(
+            wk, L.counts, steps, measure(args, hsa, L, dev, dist, world, local_rank, steps,
+                                         peaks), peaks, world)
     host = L.host
     del L, host
     torch.cuda.empty_cache()
