@@ -103,6 +103,43 @@ def test_prefix_attention(hsa, M, B, H, D, n_act, dtype, indexed):
         _check(out, ref, dtype)
 
 
+@pytest.mark.parametrize("D", [128, 64])
+def test_prefix_attention_reversed_waves(hsa, D):
+    """Enough units (8 heads x 24 query blocks = 192) that those past the first wave
+    of CTAs walk their keys backwards, starting in the ragged last tile of the second
+    source; both sources end in a ragged tile (5000 = 39 x 128 + 8 cache rows, 1500
+    = 11 x 128 + 92 fresh rows).  The oracle checks sampled rows of a head whose
+    units run forwards (0), one whose units are split between the two directions
+    (6) and one whose units all run backwards (7), with and without the split-tail
+    workspace."""
+    M, B, H, n_act = 5000, 1500, 8, 6000
+    N = M + B
+    q = synth.normal((N, H, D), 41, "bf16")
+    kc, vc = synth.normal((M, H, D), 42, "bf16"), synth.normal((M, H, D), 43, "bf16")
+    kb, vb = synth.normal((B, H, D), 44, "bf16"), synth.normal((B, H, D), 45, "bf16")
+    idx = synth.uniform_subset(N, n_act, 46)
+    k_all, v_all = torch.cat([kc, kb]), torch.cat([vc, vb])
+    g = torch.Generator().manual_seed(47)
+    rows = torch.unique(torch.cat([torch.randperm(n_act, generator=g)[:24],
+                                   torch.arange(n_act - 12, n_act), torch.arange(0, 4)]))
+    outs = []
+    for ws_on in (False, True):
+        ws = None
+        if ws_on:
+            nb = hsa.hsa_active_attention_workspace_bytes(n_act, N, H, D, 0)
+            ws = torch.empty(max(nb, 1), dtype=torch.uint8, device=DEV)
+        out = torch.full((n_act, H, D), 5.0, device=DEV).to(torch.bfloat16)
+        hsa.hsa_active_attention_prefix(q.to(DEV), idx.to(DEV), n_act, kc.to(DEV), vc.to(DEV),
+                                        kb.to(DEV), vb.to(DEV), out, workspace=ws)
+        assert hsa.hsa_get_device_error() == 0
+        outs.append(out.cpu())
+    for h in (0, 6, 7):
+        ref = oracle.attention(q[:, h:h + 1].contiguous(), k_all[:, h:h + 1].contiguous(),
+                               v_all[:, h:h + 1].contiguous(), q_idx=idx[rows])
+        for out in outs:
+            _check(out[rows, h:h + 1], ref, "bf16")
+
+
 def test_reordered_schedule_matches_full_cache(hsa):
     """T = 40 schedule with four groups.  GPU, reordered: gather of the token
     rows by `order`, prefix-only cache, scatter of the active non-baseline
