@@ -374,14 +374,17 @@ def test_attention_large_scores_rescale(hsa):
 
 @pytest.mark.parametrize("D,pos,lift", [(128, 192, 1.8), (128, 64 + 3 * 128 + 5, 1.8),
                                         (128, 739, 1.8), (128, 192, 3.0), (128, 130, 1.8),
-                                        (64, 192, 2.1), (64, 739, 2.1)])
+                                        (64, 192, 2.1), (64, 739, 2.1), (64, 739, 3.0),
+                                        (64, 700, 3.0), (128, 739, 3.0)])
 def test_attention_late_half_peak(hsa, D, pos, lift):
     """One key whose score lies 25-45 log2 units above the scores of the
     tiles before it, in the second 64-key half of a key tile (739: of the
     ragged last tile, 100 keys; 130: in a first half instead).  Against the
     running reference of the earlier tiles its probability is 2^25 to 2^45:
     below the 2^32 bound of a tile's row sum the fast path keeps those large
-    values, above it the exact path rescales; both must give the softmax."""
+    values, above it the exact path rescales O; both must give the softmax.
+    With the peak in the last key tile (lift 3) every row rescales O there,
+    the rows of the second Q tile too (300 queries: two Q tiles)."""
     N, H, n = 740, 1, 300
     u = synth.normal((1, H, D), 81)
     q = (u + 0.3 * synth.normal((n, H, D), 82)).to(torch.bfloat16)
