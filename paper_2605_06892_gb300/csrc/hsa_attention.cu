@@ -467,6 +467,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                const __grid_constant__ CUtensorMap tm_k2, const __grid_constant__ CUtensorMap tm_v2,
                const TcArgs a) {
+  // Launched with programmatic dependent launch: wait for the kernels before
+  // this one in the stream (the KV scatter writes the keys read below).  The
+  // blocks of the last wave let the next kernel start launching onto the SMs
+  // they free; no block of this grid is still waiting for an SM by then.
+  pdl_wait();
+  if (blockIdx.x + (unsigned)a.wave >= gridDim.x) pdl_trigger();
   using C = TcCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -935,6 +941,8 @@ __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float *__restrict__ ws_o, const float *__restrict__ ws_ml, int n_tail,
                     int n_whole, int pieces, int n_qblocks, int n_active, int H,
                     __nv_bfloat16 *__restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int kRows = kQT * kBM;
   const int wid = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const int u = wid / kRows, row = wid % kRows;
@@ -1180,13 +1188,15 @@ int launch_tc(const void *q, const int32_t *q_idx, int n_active, const void *k_c
   a.ws_ml = pieces > 1 ? a.ws_o + (size_t)rem * pieces * (kQT * kBM) * D : nullptr;
   const long long grid = (long long)a.n_whole + (pieces > 1 ? (long long)rem * pieces : 0);
   count_launches(1);
-  attn_tc_kernel<D><<<(unsigned)grid, kTcThreads, C::kSmem, stream>>>(mk, mv, mk2, mv2, a);
+  launch_pdl(attn_tc_kernel<D>, dim3((unsigned)grid), dim3(kTcThreads), C::kSmem, stream, mk, mv,
+             mk2, mv2, a);
   if (cudaGetLastError() != cudaSuccess) return HSA_ERR_CUDA;
   if (pieces > 1) {
     const long long warps = (long long)rem * (kQT * kBM);
     count_launches(1);
-    attn_combine_kernel<D><<<(unsigned)((warps * 32 + 255) / 256), 256, 0, stream>>>(
-        a.ws_o, a.ws_ml, rem, a.n_whole, pieces, a.n_qblocks, n_active, H, a.out);
+    launch_pdl(attn_combine_kernel<D>, dim3((unsigned)((warps * 32 + 255) / 256)), dim3(256), 0,
+               stream, (const float *)a.ws_o, (const float *)a.ws_ml, (int)rem, a.n_whole,
+               pieces, a.n_qblocks, n_active, H, a.out);
   }
   return launch_status();
 }

@@ -35,6 +35,35 @@ inline bool aligned16(const void *p) {
   return (reinterpret_cast<uintptr_t>(p) & 15u) == 0;
 }
 
+// Programmatic dependent launch, for the kernels of one HSA iteration: a
+// kernel launched with launch_pdl may be launched while the kernel before it
+// in the stream is still running.  It calls pdl_wait() before it touches
+// global memory: the wait returns once that kernel has completed and its
+// writes are visible (and, since that kernel waited the same way, every
+// earlier one).  pdl_trigger() lets the next kernel be launched; a kernel
+// that never calls it does so when its blocks exit.  Outside such a launch
+// both are no-ops.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 __device__ __forceinline__ void set_error(unsigned *err, unsigned bit) {
   atomicOr(err, bit);
 }

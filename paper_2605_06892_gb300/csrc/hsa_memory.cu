@@ -70,6 +70,8 @@ __global__ void __launch_bounds__(kThreads)
 gather_rows_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
               const int32_t *__restrict__ idx, int n_active, int N, int vecs,
               int lpr_log2, unsigned *err) {
+  pdl_wait();
+  pdl_trigger();
   copy_rows<kGatherUnroll>(n_active, vecs, lpr_log2, [&](long long j, const uint4 *&s, uint4 *&d) {
     const int r = __ldg(idx + j);
     if (r < 0 || r >= N) {
@@ -89,6 +91,8 @@ kv_scatter_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
                const uint4 *__restrict__ kf, const uint4 *__restrict__ vf,
                const int32_t *__restrict__ idx, int n_active, int N, int vecs,
                int lpr_log2, unsigned *err) {
+  pdl_wait();
+  pdl_trigger();
   copy_rows<kScatterUnroll>(2LL * n_active, vecs, lpr_log2, [&](long long jj, const uint4 *&s, uint4 *&d) {
     const bool is_v = jj >= n_active;
     const long long j = is_v ? jj - n_active : jj;
@@ -141,6 +145,8 @@ cached_euler_kernel(float4 *__restrict__ x, float4 *__restrict__ vhat,
                     const float4 *__restrict__ v_fresh, const int32_t *__restrict__ pos,
                     long long total, int vecs, int vec_shift, float dsigma, int n_fresh_rows,
                     unsigned *err) {
+  pdl_wait();
+  pdl_trigger();
   const long long stride = (long long)gridDim.x * blockDim.x;
   long long base = blockIdx.x * (long long)blockDim.x + threadIdx.x;
   int pn[kU];
@@ -506,8 +512,9 @@ extern "C" int hsa_gather_active(const void *src, size_t row_bytes, int N,
   if (!err) return HSA_ERR_CUDA;
   const int L = lanes_per_row(vecs);
   count_launches(1);
-  gather_rows_kernel<<<grid_for(n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
-      (const uint4 *)src, (uint4 *)dst, idx, n_active, N, (int)vecs, log2i(L), err);
+  launch_pdl(gather_rows_kernel, dim3(grid_for(n_active, L)), dim3(kThreads), 0,
+             (cudaStream_t)stream, (const uint4 *)src, (uint4 *)dst, idx, n_active, N, (int)vecs,
+             log2i(L), err);
   return launch_status();
 }
 
@@ -529,9 +536,9 @@ extern "C" int hsa_kv_sync_scatter(void *k_cache, void *v_cache, const void *k_f
   if (!err) return HSA_ERR_CUDA;
   const int L = lanes_per_row(vecs);
   count_launches(1);
-  kv_scatter_kernel<<<grid_for(2LL * n_active, L), kThreads, 0, (cudaStream_t)stream>>>(
-      (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh, (const uint4 *)v_fresh, idx,
-      n_active, N, (int)vecs, log2i(L), err);
+  launch_pdl(kv_scatter_kernel, dim3(grid_for(2LL * n_active, L)), dim3(kThreads), 0,
+             (cudaStream_t)stream, (uint4 *)k_cache, (uint4 *)v_cache, (const uint4 *)k_fresh,
+             (const uint4 *)v_fresh, idx, n_active, N, (int)vecs, log2i(L), err);
   return launch_status();
 }
 
@@ -558,13 +565,13 @@ extern "C" int hsa_cached_euler(float *x, float *v_cache, const float *v_fresh,
   if (blocks > cap) blocks = cap;
   count_launches(1);
   if (per == kEulerUnroll)
-    cached_euler_kernel<kEulerUnroll><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
-        (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
-        dsigma, pos ? n_fresh : 0, err);
+    launch_pdl(cached_euler_kernel<kEulerUnroll>, dim3((unsigned)blocks), dim3(kThreads), 0,
+               (cudaStream_t)stream, (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh,
+               pos, total, vecs, vec_shift, dsigma, pos ? n_fresh : 0, err);
   else
-    cached_euler_kernel<1><<<(int)blocks, kThreads, 0, (cudaStream_t)stream>>>(
-        (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh, pos, total, vecs, vec_shift,
-        dsigma, pos ? n_fresh : 0, err);
+    launch_pdl(cached_euler_kernel<1>, dim3((unsigned)blocks), dim3(kThreads), 0,
+               (cudaStream_t)stream, (float4 *)x, (float4 *)v_cache, (const float4 *)v_fresh,
+               pos, total, vecs, vec_shift, dsigma, pos ? n_fresh : 0, err);
   return launch_status();
 }
 

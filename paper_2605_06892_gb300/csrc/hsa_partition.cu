@@ -583,6 +583,8 @@ __global__ void __cluster_dims__(kCsCtas, 1, 1) __launch_bounds__(kAcThreads, 1)
 active_set_cluster_kernel(const int32_t *__restrict__ group_of, int N, int K, uint32_t mask,
                           int chunk, int32_t *__restrict__ idx, int32_t *__restrict__ pos,
                           unsigned *err) {
+  pdl_wait();
+  pdl_trigger();
   namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
   __shared__ uint32_t bits[kAcMaxChunk / 32];          // bit t: token lo + t is active
@@ -808,8 +810,8 @@ extern "C" int hsa_partition_active(const int32_t *group_of, int N, int T, const
   if (N <= kAcMaxN && cluster_active_ready()) {
     const int chunk = (N + kCsCtas - 1) / kCsCtas;
     count_launches(1);
-    active_set_cluster_kernel<<<kCsCtas, kAcThreads, 0, s>>>(group_of, N, K, mask, chunk, idx,
-                                                             pos, err);
+    launch_pdl(active_set_cluster_kernel, dim3(kCsCtas), dim3(kAcThreads), 0, s, group_of, N, K,
+               mask, chunk, idx, pos, err);
     return launch_status();
   }
   // Larger layers: chunks of whole 1024-token rounds, at most one block per
